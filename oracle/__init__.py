@@ -1,0 +1,20 @@
+"""CPU oracle for the low-bit MLA decode path (test infrastructure).
+
+This package is the independent, slow, obviously-correct definition that the
+CUDA library is checked against. It is test infrastructure: only ``tests/``,
+``__graft_entry__.smoke()`` and the CPU-baseline leg of ``bench.py`` may import
+or run it. The product path never calls it, and it shares no code, constants
+or helpers with ``paper_2609_36760_gb300``.
+
+Modules
+-------
+quantizer  per-token group-64 asymmetric quantiser and bit packing (App. C.4)
+layout     this library's 64-token block byte layout, writer and reader
+attention  dequantisation, absorbed MLA decode attention in fp64 (Eq. mla_compact)
+           and the split-result merge (App. C.5, global attention normalisation)
+storage    the persistent-storage closed form (App. C.5, Eq. physical_cache_storage)
+
+Every function is pinned by tests under ``tests/test_oracle_*.py``; nothing in
+this package is marked "parity unpinned".
+"""
+from . import attention, layout, quantizer, storage  # noqa: F401
