@@ -1,0 +1,177 @@
+/*
+ * qmla — low-bit MLA decode attention on one GB300 (sm_103a).
+ *
+ * C ABI of the library libqmla.so. It implements the decode hot path of
+ * QuantMLA (arXiv 2609.36760): Multi-head Latent Attention read directly from a
+ * jointly low-bit paged cache, with unpacking and dequantisation fused into the
+ * attention (Sec. 3.3; App. C.5).
+ *
+ *   qmla_quant_append   quantise + pack new tokens into the paged cache
+ *                       (App. C.4 quantiser; App. C.5 "cache update": content- and
+ *                       RoPE-cache quantisation, integer packing, slot-mapped
+ *                       page insertion)
+ *   qmla_mla_decode     split-KV decode attention over the packed cache, plus the
+ *                       split-result combination (Eq. mla_compact; App. C.5
+ *                       "global attention normalization")
+ *
+ * Conventions for every call
+ * --------------------------
+ * - Pointers named *_dev are device pointers owned by the caller; the library
+ *   never allocates, frees or keeps them. Host pointers are marked _host.
+ * - Every call that launches work is asynchronous on `stream` (a cudaStream_t;
+ *   NULL = legacy default stream) and returns a status code immediately.
+ *   Arguments are validated on the host before anything is launched; an invalid
+ *   argument launches nothing.
+ * - Problems only visible on the device (a bad block id, a position beyond the
+ *   block table, a pipeline wait that ran out) are OR-ed into the caller's
+ *   32-bit error word `dev_err_dev` (QMLA_DEVERR_*). The offending access is
+ *   skipped; no call traps or aborts. Read the word with qmla_read_dev_err.
+ * - bf16 / fp16 tensors are passed as uint16_t bit patterns.
+ *
+ * Cache format (this library's own 64-token block, little-endian)
+ * ----------------------------------------------------------------
+ * Each token is quantised in 9 groups of 64 coordinates: groups 0..7 are the
+ * content latent c_KV channels [64g, 64g+64) at c_bits (4 or 2), group 8 is the
+ * decoupled RoPE key k_pe (d_r = 64) at 4 bits. Per group, per token
+ * (App. C.4, with the fp16 staging fixed by this library):
+ *     d = RN_f32(x_max - x_min);  s = RN_f16(RN_f32(max(d, 1e-8) / m)), m = 2^b - 1
+ *     (s = 2^-24 if that underflows to 0, 65504 if it overflows)
+ *     z = clip(rne(-x_min / s), 0, m);  q = clip(rne(x / s + z), 0, m)
+ * Codes are packed low bits first: INT4 byte j = q[2j] | q[2j+1] << 4, INT2
+ * byte j = q[4j] | q[4j+1] << 2 | q[4j+2] << 4 | q[4j+3] << 6.
+ * A block of 64 token slots, cb = 64 * c_bits / 8:
+ *     [0, 8*64*cb)                 content codes   [group 8][slot 64][cb bytes]
+ *     [8*64*cb, +2048)             RoPE-key codes  [slot 64][32 bytes]
+ *     [8*64*cb + 2048, +2304)      scale/zero      [group 9][slot 64][fp16 s, fp16 z]
+ * INT4 content: 20736 bytes per block; INT2 content: 12544 bytes per block.
+ * Token at position p of sequence b lives in block block_table[b*max_blocks + p/64],
+ * slot p % 64.
+ *
+ * The BF16 comparison cache (qmla_bf16_append / qmla_mla_decode_bf16cache)
+ * stores each token as 576 bf16 (latent then k_pe): blocks of 64 x 1152 bytes,
+ * the paper's BF16 page (App. C.5, storage layout).
+ */
+#ifndef QMLA_H_
+#define QMLA_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* qmla_stream_t; /* same type as cudaStream_t */
+
+/* Status codes returned by every call. */
+enum qmla_status {
+  QMLA_OK = 0,
+  QMLA_ERR_INVALID_ARG = 1,          /* null pointer, bad size, bad bit width, misalignment */
+  QMLA_ERR_UNSUPPORTED = 2,          /* no sm_103a device, or a shape outside the supported range */
+  QMLA_ERR_WORKSPACE_TOO_SMALL = 3,  /* decode workspace smaller than qmla_decode_workspace_bytes */
+  QMLA_ERR_CUDA = 4                  /* a CUDA runtime call failed; see qmla_last_cuda_error */
+};
+
+/* Bits of the device error word. */
+enum qmla_device_error {
+  QMLA_DEVERR_BAD_BLOCK = 1u,     /* a block-table entry outside [0, num_blocks) was needed */
+  QMLA_DEVERR_BAD_POSITION = 2u,  /* a position or sequence length < 0 or beyond max_blocks*64 */
+  QMLA_DEVERR_BAD_SEQ = 4u,       /* an append sequence id outside [0, num_seqs) */
+  QMLA_DEVERR_TIMEOUT = 8u        /* an on-chip pipeline wait ran out; that kernel left early */
+};
+
+/* Bytes of one 64-token block for content bit width c_bits (4 -> 20736,
+ * 2 -> 12544); 0 if c_bits is not supported. */
+size_t qmla_block_bytes(int c_bits);
+
+/* Bytes of one 64-token BF16 comparison block (73728). */
+size_t qmla_bf16_block_bytes(void);
+
+/*
+ * Quantise n new tokens and insert them into the packed cache
+ * (App. C.4 quantiser; App. C.5 fused writer without the BF16 protection
+ * buffers).
+ *
+ *   pool_dev        [num_blocks * qmla_block_bytes(c_bits)] bytes, 16-byte aligned;
+ *                   only the slots of the given tokens are written
+ *   c_bits          content bit width, 4 or 2 (the RoPE key is always 4-bit)
+ *   latent_dev      [n, 512] bf16, row-major, 4-byte aligned: content latent c_KV
+ *   k_pe_dev        [n, 64]  bf16, row-major, 4-byte aligned: decoupled RoPE key
+ *   seq_ids_dev     [n] int32 sequence of each token, or NULL meaning token i
+ *                   belongs to sequence i
+ *   positions_dev   [n] int32 zero-based position of each token in its sequence
+ *   block_table_dev [num_seqs, max_blocks] int32 physical block ids
+ *   dev_err_dev     device error word (see above)
+ * Two tokens with the same (sequence, position) in one call race; the result
+ * is one of them. n == 0 is a no-op.
+ */
+int qmla_quant_append(void* pool_dev, int c_bits, int num_blocks, const uint16_t* latent_dev,
+                      const uint16_t* k_pe_dev, const int32_t* seq_ids_dev,
+                      const int32_t* positions_dev, int n, const int32_t* block_table_dev,
+                      int num_seqs, int max_blocks, uint32_t* dev_err_dev, qmla_stream_t stream);
+
+/* Same insertion into the BF16 comparison cache (blocks of qmla_bf16_block_bytes()):
+ * the 576 bf16 values of each token are copied unchanged. */
+int qmla_bf16_append(void* pool_dev, int num_blocks, const uint16_t* latent_dev,
+                     const uint16_t* k_pe_dev, const int32_t* seq_ids_dev,
+                     const int32_t* positions_dev, int n, const int32_t* block_table_dev,
+                     int num_seqs, int max_blocks, uint32_t* dev_err_dev, qmla_stream_t stream);
+
+/* Workspace bytes qmla_mla_decode needs for this batch and head count on the
+ * current device (split plan + split partials). */
+size_t qmla_decode_workspace_bytes(int batch, int heads);
+
+/*
+ * Decode attention of one query token per sequence over the packed cache
+ * (Eq. mla_compact with the dequantised cache s (q - z), App. C.4):
+ *     S[b,h,t] = softmax_scale * (q_latent[b,h,:] . C_hat[b,t,:] + q_pe[b,h,:] . K_hat[b,t,:])
+ *     out[b,h,:] = sum_t softmax_t(S[b,h,:]) C_hat[b,t,:]      (t < seq_lens[b])
+ *     lse[b,h]   = log sum_t exp(S[b,h,t])
+ * The caller applies the value/output up-projection. Sequences are split
+ * across the GPU's SMs and the split results merged with the App. C.5 rule.
+ *
+ *   pool_dev        packed cache written by qmla_quant_append with the same c_bits
+ *   q_latent_dev    [batch, heads, 512] bf16 absorbed content query, 16-byte aligned
+ *   q_pe_dev        [batch, heads, 64]  bf16 RoPE query, 16-byte aligned
+ *   heads           1..128
+ *   block_table_dev [batch, max_blocks] int32
+ *   seq_lens_dev    [batch] int32 tokens to attend to (including any just appended)
+ *   softmax_scale   tau, e.g. 1/sqrt(192)
+ *   out_dev         [batch, heads, 512] float32
+ *   lse_dev         [batch, heads] float32 natural-log LSE, or NULL
+ *   workspace_dev   >= qmla_decode_workspace_bytes(batch, heads) bytes, 256-byte aligned;
+ *                   contents need no initialisation and are scratch after the call
+ * A sequence with seq_lens == 0 gets out = 0 and lse = -inf.
+ */
+int qmla_mla_decode(const void* pool_dev, int c_bits, int num_blocks, const uint16_t* q_latent_dev,
+                    const uint16_t* q_pe_dev, int batch, int heads, const int32_t* block_table_dev,
+                    int max_blocks, const int32_t* seq_lens_dev, float softmax_scale,
+                    float* out_dev, float* lse_dev, void* workspace_dev, size_t workspace_bytes,
+                    uint32_t* dev_err_dev, qmla_stream_t stream);
+
+/* The same decode over the BF16 comparison cache (same kernel, no dequantisation;
+ * the paper's BF16 baseline, App. F.1). */
+int qmla_mla_decode_bf16cache(const void* pool_dev, int num_blocks, const uint16_t* q_latent_dev,
+                              const uint16_t* q_pe_dev, int batch, int heads,
+                              const int32_t* block_table_dev, int max_blocks,
+                              const int32_t* seq_lens_dev, float softmax_scale, float* out_dev,
+                              float* lse_dev, void* workspace_dev, size_t workspace_bytes,
+                              uint32_t* dev_err_dev, qmla_stream_t stream);
+
+/* Copies the device error word to *host_out after synchronising `stream`. */
+int qmla_read_dev_err(const uint32_t* dev_err_dev, uint32_t* host_out, qmla_stream_t stream);
+
+/* The cudaError_t of the last failed CUDA call in this thread (0 if none). */
+int qmla_last_cuda_error(void);
+
+/* Static text for a status code. */
+const char* qmla_status_string(int status);
+
+/* Number of SMs of the current device (the decode grid size), or -1. */
+int qmla_num_sms(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* QMLA_H_ */

@@ -1,0 +1,197 @@
+// Host side of the C ABI declared in include/qmla.h: argument validation,
+// device checks and kernel launches. Nothing here allocates device memory.
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "qmla.h"
+
+namespace {
+
+thread_local int g_last_cuda_error = 0;
+
+int cuda_fail(cudaError_t e) {
+  g_last_cuda_error = static_cast<int>(e);
+  return QMLA_ERR_CUDA;
+}
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+// SM count and architecture of each device, looked up once.
+struct DevInfo {
+  int sms = -1;
+  bool supported = false;
+};
+DevInfo g_dev[64];
+
+int current_device_info(DevInfo& out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e);
+  if (dev < 0 || dev >= 64) return QMLA_ERR_UNSUPPORTED;
+  if (g_dev[dev].sms < 0) {
+    int major = 0, minor = 0, sms = 0;
+    if ((e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev)) != cudaSuccess) return cuda_fail(e);
+    if ((e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev)) != cudaSuccess) return cuda_fail(e);
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return cuda_fail(e);
+    g_dev[dev].supported = (major == 10 && minor == 3);
+    g_dev[dev].sms = sms;
+  }
+  out = g_dev[dev];
+  return out.supported ? QMLA_OK : QMLA_ERR_UNSUPPORTED;
+}
+
+int append_common_checks(const void* pool, int num_blocks, const uint16_t* latent, const uint16_t* k_pe,
+                         const int32_t* positions, int n, const int32_t* table, int num_seqs,
+                         int max_blocks) {
+  if (n < 0 || num_blocks <= 0 || num_seqs <= 0 || max_blocks <= 0) return QMLA_ERR_INVALID_ARG;
+  if (n == 0) return QMLA_OK;
+  if (pool == nullptr || latent == nullptr || k_pe == nullptr || positions == nullptr || table == nullptr)
+    return QMLA_ERR_INVALID_ARG;
+  if (!aligned(pool, 16) || !aligned(latent, 4) || !aligned(k_pe, 4) || !aligned(positions, 4) ||
+      !aligned(table, 4))
+    return QMLA_ERR_INVALID_ARG;
+  if (static_cast<long long>(max_blocks) * qmla::kBlockTokens > INT32_MAX) return QMLA_ERR_INVALID_ARG;
+  return QMLA_OK;
+}
+
+int decode_common(const void* pool, int kind, int num_blocks, const uint16_t* q_latent, const uint16_t* q_pe,
+                  int batch, int heads, const int32_t* table, int max_blocks, const int32_t* seq_lens,
+                  float softmax_scale, float* out, float* lse, void* workspace, size_t workspace_bytes,
+                  uint32_t* dev_err, qmla_stream_t stream) {
+  if (pool == nullptr || q_latent == nullptr || q_pe == nullptr || table == nullptr || seq_lens == nullptr ||
+      out == nullptr || workspace == nullptr)
+    return QMLA_ERR_INVALID_ARG;
+  if (batch <= 0 || heads < 1 || heads > 128 || num_blocks <= 0 || max_blocks <= 0) return QMLA_ERR_INVALID_ARG;
+  if (!(softmax_scale > 0.0f) || softmax_scale > 1e30f) return QMLA_ERR_INVALID_ARG;
+  if (!aligned(pool, 16) || !aligned(q_latent, 16) || !aligned(q_pe, 16) || !aligned(table, 4) ||
+      !aligned(seq_lens, 4) || !aligned(out, 16) || (lse != nullptr && !aligned(lse, 4)) ||
+      !aligned(workspace, 256))
+    return QMLA_ERR_INVALID_ARG;
+  if (static_cast<long long>(max_blocks) * qmla::kBlockTokens > INT32_MAX) return QMLA_ERR_INVALID_ARG;
+  DevInfo di;
+  int st = current_device_info(di);
+  if (st != QMLA_OK) return st;
+  const qmla::DecodeWorkspace w = qmla::decode_workspace_layout(batch, heads, di.sms);
+  if (workspace_bytes < w.total) return QMLA_ERR_WORKSPACE_TOO_SMALL;
+  qmla::DecodeArgs a;
+  a.pool = pool;
+  a.cache_kind = kind;
+  a.num_blocks = num_blocks;
+  a.q_latent = q_latent;
+  a.q_pe = q_pe;
+  a.batch = batch;
+  a.heads = heads;
+  a.table = table;
+  a.max_blocks = max_blocks;
+  a.seq_lens = seq_lens;
+  a.softmax_scale = softmax_scale;
+  a.out = out;
+  a.lse = lse;
+  a.workspace = workspace;
+  a.dev_err = dev_err;
+  a.grid = di.sms;
+  cudaError_t e = qmla::launch_decode(a, reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t qmla_block_bytes(int c_bits) {
+  if (c_bits == 4) return qmla::BlockLayout<4>::kBytes;
+  if (c_bits == 2) return qmla::BlockLayout<2>::kBytes;
+  return 0;
+}
+
+size_t qmla_bf16_block_bytes(void) { return qmla::kBf16BlockBytes; }
+
+int qmla_quant_append(void* pool_dev, int c_bits, int num_blocks, const uint16_t* latent_dev,
+                      const uint16_t* k_pe_dev, const int32_t* seq_ids_dev, const int32_t* positions_dev,
+                      int n, const int32_t* block_table_dev, int num_seqs, int max_blocks,
+                      uint32_t* dev_err_dev, qmla_stream_t stream) {
+  if (c_bits != 4 && c_bits != 2) return QMLA_ERR_INVALID_ARG;
+  int st = append_common_checks(pool_dev, num_blocks, latent_dev, k_pe_dev, positions_dev, n, block_table_dev,
+                                num_seqs, max_blocks);
+  if (st != QMLA_OK || n == 0) return st;
+  DevInfo di;
+  if ((st = current_device_info(di)) != QMLA_OK) return st;
+  cudaError_t e = qmla::launch_quant_append(pool_dev, c_bits, num_blocks, latent_dev, k_pe_dev, seq_ids_dev,
+                                            positions_dev, n, block_table_dev, num_seqs, max_blocks,
+                                            dev_err_dev, reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
+}
+
+int qmla_bf16_append(void* pool_dev, int num_blocks, const uint16_t* latent_dev, const uint16_t* k_pe_dev,
+                     const int32_t* seq_ids_dev, const int32_t* positions_dev, int n,
+                     const int32_t* block_table_dev, int num_seqs, int max_blocks, uint32_t* dev_err_dev,
+                     qmla_stream_t stream) {
+  int st = append_common_checks(pool_dev, num_blocks, latent_dev, k_pe_dev, positions_dev, n, block_table_dev,
+                                num_seqs, max_blocks);
+  if (st != QMLA_OK || n == 0) return st;
+  DevInfo di;
+  if ((st = current_device_info(di)) != QMLA_OK) return st;
+  cudaError_t e = qmla::launch_bf16_append(pool_dev, num_blocks, latent_dev, k_pe_dev, seq_ids_dev, positions_dev,
+                                           n, block_table_dev, num_seqs, max_blocks, dev_err_dev,
+                                           reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
+}
+
+size_t qmla_decode_workspace_bytes(int batch, int heads) {
+  if (batch <= 0 || heads < 1 || heads > 128) return 0;
+  DevInfo di;
+  if (current_device_info(di) != QMLA_OK) return 0;
+  return qmla::decode_workspace_layout(batch, heads, di.sms).total;
+}
+
+int qmla_mla_decode(const void* pool_dev, int c_bits, int num_blocks, const uint16_t* q_latent_dev,
+                    const uint16_t* q_pe_dev, int batch, int heads, const int32_t* block_table_dev, int max_blocks,
+                    const int32_t* seq_lens_dev, float softmax_scale, float* out_dev, float* lse_dev,
+                    void* workspace_dev, size_t workspace_bytes, uint32_t* dev_err_dev, qmla_stream_t stream) {
+  if (c_bits != 4 && c_bits != 2) return QMLA_ERR_INVALID_ARG;
+  return decode_common(pool_dev, c_bits, num_blocks, q_latent_dev, q_pe_dev, batch, heads, block_table_dev,
+                       max_blocks, seq_lens_dev, softmax_scale, out_dev, lse_dev, workspace_dev, workspace_bytes,
+                       dev_err_dev, stream);
+}
+
+int qmla_mla_decode_bf16cache(const void* pool_dev, int num_blocks, const uint16_t* q_latent_dev,
+                              const uint16_t* q_pe_dev, int batch, int heads, const int32_t* block_table_dev,
+                              int max_blocks, const int32_t* seq_lens_dev, float softmax_scale, float* out_dev,
+                              float* lse_dev, void* workspace_dev, size_t workspace_bytes, uint32_t* dev_err_dev,
+                              qmla_stream_t stream) {
+  return decode_common(pool_dev, 16, num_blocks, q_latent_dev, q_pe_dev, batch, heads, block_table_dev, max_blocks,
+                       seq_lens_dev, softmax_scale, out_dev, lse_dev, workspace_dev, workspace_bytes, dev_err_dev,
+                       stream);
+}
+
+int qmla_read_dev_err(const uint32_t* dev_err_dev, uint32_t* host_out, qmla_stream_t stream) {
+  if (dev_err_dev == nullptr || host_out == nullptr) return QMLA_ERR_INVALID_ARG;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMemcpyAsync(host_out, dev_err_dev, sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
+}
+
+int qmla_last_cuda_error(void) { return g_last_cuda_error; }
+
+const char* qmla_status_string(int status) {
+  switch (status) {
+    case QMLA_OK: return "ok";
+    case QMLA_ERR_INVALID_ARG: return "invalid argument";
+    case QMLA_ERR_UNSUPPORTED: return "unsupported device or shape";
+    case QMLA_ERR_WORKSPACE_TOO_SMALL: return "workspace too small";
+    case QMLA_ERR_CUDA: return "CUDA error";
+    default: return "unknown status";
+  }
+}
+
+int qmla_num_sms(void) {
+  DevInfo di;
+  if (current_device_info(di) != QMLA_OK) return -1;
+  return di.sms;
+}
+
+}  // extern "C"

@@ -1,0 +1,166 @@
+// Quantise-and-pack cache writer (App. C.4 quantiser; App. C.5 cache update:
+// content- and RoPE-cache quantisation, integer packing and slot-mapped page
+// insertion), and the plain BF16 writer for the comparison cache.
+//
+// One warp per token. For each of the 9 groups of 64 coordinates, lane l holds
+// coordinates 2l and 2l+1; the group extrema come from warp reductions, every
+// lane quantises its two values, and the packed code words are assembled with
+// shuffles and stored by the lanes that own them.
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace qmla {
+namespace {
+
+__device__ __forceinline__ float warp_min_f32(float v) {
+  float r;
+  asm volatile("redux.sync.min.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(v));
+  return r;
+}
+__device__ __forceinline__ float warp_max_f32(float v) {
+  float r;
+  asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(v));
+  return r;
+}
+
+// Stored fp16 scale and integer zero point of one group (App. C.4 with the
+// fp16 staging of include/qmla.h): s = RN_f16(RN_f32(max(d, 1e-8) / m)),
+// clamped to [2^-24, 65504]; z = clip(rne(-x_min / s), 0, m).
+__device__ __forceinline__ void group_scale(float xmin, float xmax, int m, float& s, float& z) {
+  const float d = xmax - xmin;
+  const float s32 = __fdiv_rn(fmaxf(d, 1e-8f), static_cast<float>(m));
+  s = __half2float(__float2half_rn(s32));
+  if (s == 0.0f) s = 5.9604644775390625e-08f;  // 2^-24, the smallest fp16 subnormal
+  if (isinf(s)) s = 65504.0f;
+  z = fminf(fmaxf(rintf(__fdiv_rn(-xmin, s)), 0.0f), static_cast<float>(m));
+}
+
+__device__ __forceinline__ uint32_t quant_code(float x, float s, float z, int m) {
+  // q = clip(rne(x / s + z), 0, m): z is added before rounding.
+  return static_cast<uint32_t>(fminf(fmaxf(rintf(__fdiv_rn(x, s) + z), 0.0f), static_cast<float>(m)));
+}
+
+// Looks up and validates the destination of token i. Returns null (after
+// recording the error) when the token cannot be written.
+__device__ __forceinline__ uint8_t* token_block(uint8_t* pool, size_t block_bytes, int num_blocks,
+                                                const int32_t* seq_ids, const int32_t* positions,
+                                                int i, const int32_t* table, int num_seqs,
+                                                int max_blocks, uint32_t* dev_err, int& slot) {
+  const int seq = seq_ids != nullptr ? seq_ids[i] : i;
+  const int pos = positions[i];
+  if (seq < 0 || seq >= num_seqs) {
+    report(dev_err, QMLA_DEVERR_BAD_SEQ);
+    return nullptr;
+  }
+  if (pos < 0 || pos >= max_blocks * kBlockTokens) {
+    report(dev_err, QMLA_DEVERR_BAD_POSITION);
+    return nullptr;
+  }
+  const int blk = table[static_cast<size_t>(seq) * max_blocks + pos / kBlockTokens];
+  if (blk < 0 || blk >= num_blocks) {
+    report(dev_err, QMLA_DEVERR_BAD_BLOCK);
+    return nullptr;
+  }
+  slot = pos % kBlockTokens;
+  return pool + static_cast<size_t>(blk) * block_bytes;
+}
+
+template <int CB>
+__global__ void __launch_bounds__(256) quant_append_kernel(
+    uint8_t* __restrict__ pool, int num_blocks, const __nv_bfloat162* __restrict__ latent,
+    const __nv_bfloat162* __restrict__ k_pe, const int32_t* __restrict__ seq_ids,
+    const int32_t* __restrict__ positions, int n, const int32_t* __restrict__ table, int num_seqs,
+    int max_blocks, uint32_t* dev_err) {
+  using L = BlockLayout<CB>;
+  const int tok = static_cast<int>((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  const int lane = threadIdx.x & 31;
+  if (tok >= n) return;
+  int slot = 0;
+  uint8_t* blk = token_block(pool, L::kBytes, num_blocks, seq_ids, positions, tok, table, num_seqs,
+                             max_blocks, lane == 0 ? dev_err : nullptr, slot);
+  if (blk == nullptr) return;
+
+#pragma unroll 1
+  for (int g = 0; g < kGroups; ++g) {
+    const int bits = g < 8 ? CB : kPeBits;
+    const int m = (1 << bits) - 1;
+    const __nv_bfloat162 v = g < 8 ? latent[static_cast<size_t>(tok) * (kDc / 2) + g * 32 + lane]
+                                   : k_pe[static_cast<size_t>(tok) * (kDr / 2) + lane];
+    const float x0 = __low2float(v), x1 = __high2float(v);
+    const float xmin = warp_min_f32(fminf(x0, x1));
+    const float xmax = warp_max_f32(fmaxf(x0, x1));
+    float s, z;
+    group_scale(xmin, xmax, m, s, z);
+    const uint32_t code = quant_code(x0, s, z, m) | (quant_code(x1, s, z, m) << bits);
+    // Lane l's 2*bits bits sit at bit offset 2*bits*l of the group's code string.
+    const int lane_bits = 2 * bits;
+    const int lanes_per_word = 32 / lane_bits;
+    uint32_t word = code << ((lane % lanes_per_word) * lane_bits);
+    for (int off = 1; off < lanes_per_word; off <<= 1) word |= __shfl_xor_sync(0xffffffffu, word, off);
+    if (lane % lanes_per_word == 0) {
+      reinterpret_cast<uint32_t*>(blk + L::code_off(g, slot))[lane / lanes_per_word] = word;
+    }
+    if (lane == 0) {
+      *reinterpret_cast<__half2*>(blk + L::sz_off(g, slot)) =
+          __halves2half2(__float2half_rn(s), __float2half_rn(z));
+    }
+  }
+}
+
+__global__ void __launch_bounds__(256) bf16_append_kernel(
+    uint8_t* __restrict__ pool, int num_blocks, const uint32_t* __restrict__ latent,
+    const uint32_t* __restrict__ k_pe, const int32_t* __restrict__ seq_ids,
+    const int32_t* __restrict__ positions, int n, const int32_t* __restrict__ table, int num_seqs,
+    int max_blocks, uint32_t* dev_err) {
+  const int tok = static_cast<int>((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  const int lane = threadIdx.x & 31;
+  if (tok >= n) return;
+  int slot = 0;
+  uint8_t* blk = token_block(pool, kBf16BlockBytes, num_blocks, seq_ids, positions, tok, table,
+                             num_seqs, max_blocks, lane == 0 ? dev_err : nullptr, slot);
+  if (blk == nullptr) return;
+  uint32_t* dst = reinterpret_cast<uint32_t*>(blk + slot * kDqk * 2);
+  for (int w = lane; w < kDc / 2; w += 32) dst[w] = latent[static_cast<size_t>(tok) * (kDc / 2) + w];
+  dst[kDc / 2 + lane] = k_pe[static_cast<size_t>(tok) * (kDr / 2) + lane];
+}
+
+}  // namespace
+
+cudaError_t launch_quant_append(void* pool, int c_bits, int num_blocks, const uint16_t* latent,
+                                const uint16_t* k_pe, const int32_t* seq_ids,
+                                const int32_t* positions, int n, const int32_t* table, int num_seqs,
+                                int max_blocks, uint32_t* dev_err, cudaStream_t stream) {
+  if (n == 0) return cudaSuccess;
+  const dim3 block(256);
+  const dim3 grid(static_cast<unsigned>((static_cast<long long>(n) * 32 + 255) / 256));
+  auto* lat = reinterpret_cast<const __nv_bfloat162*>(latent);
+  auto* kp = reinterpret_cast<const __nv_bfloat162*>(k_pe);
+  if (c_bits == 4) {
+    quant_append_kernel<4><<<grid, block, 0, stream>>>(static_cast<uint8_t*>(pool), num_blocks, lat,
+                                                       kp, seq_ids, positions, n, table, num_seqs,
+                                                       max_blocks, dev_err);
+  } else {
+    quant_append_kernel<2><<<grid, block, 0, stream>>>(static_cast<uint8_t*>(pool), num_blocks, lat,
+                                                       kp, seq_ids, positions, n, table, num_seqs,
+                                                       max_blocks, dev_err);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bf16_append(void* pool, int num_blocks, const uint16_t* latent,
+                               const uint16_t* k_pe, const int32_t* seq_ids,
+                               const int32_t* positions, int n, const int32_t* table, int num_seqs,
+                               int max_blocks, uint32_t* dev_err, cudaStream_t stream) {
+  if (n == 0) return cudaSuccess;
+  const dim3 block(256);
+  const dim3 grid(static_cast<unsigned>((static_cast<long long>(n) * 32 + 255) / 256));
+  bf16_append_kernel<<<grid, block, 0, stream>>>(
+      static_cast<uint8_t*>(pool), num_blocks, reinterpret_cast<const uint32_t*>(latent),
+      reinterpret_cast<const uint32_t*>(k_pe), seq_ids, positions, n, table, num_seqs, max_blocks,
+      dev_err);
+  return cudaGetLastError();
+}
+
+}  // namespace qmla

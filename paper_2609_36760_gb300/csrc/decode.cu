@@ -1,0 +1,917 @@
+// Split-KV MLA decode over the low-bit paged cache (Eq. mla_compact; App. C.5
+// "cache update and tile reuse" and "global attention normalization").
+//
+// Three kernels run per decode call:
+//   plan_kernel    per-sequence tile counts -> prefix over (sequence, head group)
+//                  units; the flattened tile list is cut into one equal range per
+//                  SM ("metadata construction", App. F.1).
+//   decode_main    one persistent CTA per SM walks its tile range. A tile is 128
+//                  cached tokens (two 64-token blocks) for one head group of HG
+//                  heads. Per tile:
+//                    dequant warps  gather packed codes + fp16 (s, z) from global
+//                                   memory (prefetched a tile ahead), unpack and
+//                                   dequantise RN_f16(s (q - z)) into nine
+//                                   swizzled fp16 chunks of 128 tokens x 64
+//                                   channels in shared memory;
+//                    MMA thread     S^T[t,h] = C_hat[t,:] . q[h,:] over 576
+//                                   channels (tcgen05, M=128 tokens, N=HG,
+//                                   K-major A and B) into TMEM;
+//                    softmax warps  read S^T from TMEM (one token per thread),
+//                                   keep a per-head reference max (rescaling O
+//                                   only when a score exceeds it by 2^8), write
+//                                   P^T = 2^(S*scale*log2e - m) as fp16;
+//                    MMA thread     O^T[c,h] += C_hat[:,c]^T P^T (M = 128
+//                                   channels x 4, N=HG, K = 128 tokens; the same
+//                                   shared-memory chunks read MN-major).
+//                  The reconstructed content tile serves both QK and PV and a
+//                  chunk is overwritten only after the PV that reads it commits.
+//                  At a segment end the softmax warps write the final output, or
+//                  an unnormalised partial (m, l, o) when the unit is split.
+//   combine_kernel merges the partials of split units with
+//                  m = max m_j, l = sum e^(m_j - m) l_j, O = sum e^(m_j - m) o_j / l.
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace qmla {
+namespace {
+
+constexpr int kTileTokens = 128;                 // tokens per tile (M of QK)
+constexpr int kChunkBytes = kTileTokens * 128;   // 128 tokens x 64 fp16 channels
+constexpr int kNumChunks = 9;                    // 8 content chunks + RoPE-key chunk
+constexpr int kNumDqWarps = 8;
+constexpr int kSmWarp0 = kNumDqWarps;            // softmax warps 8..11 (TMEM lane quarters 0..3)
+constexpr int kMmaWarp = kNumDqWarps + 4;        // warp 12 issues MMAs and owns TMEM
+constexpr int kThreads = (kMmaWarp + 1) * 32;    // 416
+constexpr uint64_t kWaitNs = 2000000000ull;      // bound of every on-chip wait (2 s)
+constexpr float kRescaleLog2 = 8.0f;             // rescale O only above 2^8 growth
+constexpr float kLn2 = 0.6931471805599453f;
+
+struct Params {
+  const uint8_t* pool;
+  int num_blocks;
+  const __nv_bfloat16* q_lat;
+  const __nv_bfloat16* q_pe;
+  int batch, heads, n_hg;
+  const int32_t* table;
+  int max_blocks;
+  const int32_t* seq_lens;
+  float scale_log2;  // softmax_scale * log2(e)
+  float* out;
+  float* lse;
+  const int32_t* prefix;
+  int32_t* prefix_w;
+  float* part_o;   // [(grid + units)][HG][512]
+  float* part_ml;  // [(grid + units)][HG][2]
+  uint32_t* dev_err;
+  int grid;
+};
+
+struct __align__(16) Ctrl {
+  uint64_t full[kNumChunks];
+  uint64_t empty[kNumChunks];
+  uint64_t s_full, p_full, pv_done, o_free, q_empty, q_full, fin;
+  uint64_t grp[3];
+  uint32_t tmem_base;
+  uint32_t abort;
+  uint32_t vote[2][4];
+  float m_ref[64];
+  float alpha[64];
+  float red[4][64];
+};
+
+template <int HG>
+struct Cfg {
+  static constexpr int kQBytes = kNumChunks * HG * 128;
+  static constexpr uint32_t kTmemCols = HG == 64 ? 512 : (HG == 32 ? 256 : 128);
+  static constexpr int kSmem = 1024 + kNumChunks * kChunkBytes + kQBytes + (int)sizeof(Ctrl);
+  static constexpr uint32_t kPRowBytes = 2 * HG;  // P^T tile row (one token, HG fp16)
+};
+
+// Channel order inside each 8-channel (16-byte) piece of a reconstructed row:
+// the unpacking below yields nibble/crumb pairs in this order, and the query
+// tile and the output mapping use the same permutation.
+template <int CB>
+struct Perm {
+  // position p of a piece holds channel at(p): INT4 swaps bits 0 and 1 of p
+  // ([0,2,1,3,4,6,5,7]); INT2 rotates them ([0,4,1,5,2,6,3,7]); BF16 keeps p.
+  __host__ __device__ static constexpr int at(int p) {
+    if constexpr (CB == 4) {
+      return (p & 4) | ((p & 1) << 1) | ((p >> 1) & 1);
+    } else if constexpr (CB == 2) {
+      return ((p & 1) << 2) | (p >> 1);
+    } else {
+      return p;
+    }
+  }
+};
+static_assert(Perm<4>::at(1) == 2 && Perm<4>::at(2) == 1 && Perm<4>::at(5) == 6 && Perm<4>::at(7) == 7, "INT4 order");
+static_assert(Perm<2>::at(1) == 4 && Perm<2>::at(2) == 1 && Perm<2>::at(6) == 3 && Perm<2>::at(7) == 7, "INT2 order");
+
+// --------------------------------------------------------------- helpers
+__device__ __forceinline__ uint4 ldg_nc_v4(const void* ptr) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(ptr));
+  return r;
+}
+__device__ __forceinline__ uint32_t ldg_nc_u32(const void* ptr) {
+  uint32_t r;
+  asm volatile("ld.global.nc.L1::no_allocate.u32 %0, [%1];" : "=r"(r) : "l"(ptr));
+  return r;
+}
+__device__ __forceinline__ void sts_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
+               : "memory");
+}
+// RN_f16((x - zz) * s) per half: the subtraction of two integers below 2048 is
+// exact, so this is a single rounding of s (q - z).
+__device__ __forceinline__ uint32_t dq2(uint32_t x, uint32_t zz, uint32_t ss) {
+  uint32_t t, r;
+  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(t) : "r"(x), "r"(zz));
+  asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(t), "r"(ss));
+  return r;
+}
+__device__ __forceinline__ uint32_t pack_h2(float lo, float hi) {
+  const __half2 h = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+__device__ __forceinline__ float warp_max_f32(float v) {
+  float r;
+  asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(v));
+  return r;
+}
+
+// Wait sites, reported in bits 8.. of the error word when a wait runs out.
+enum WaitSite : uint32_t {
+  kSiteDqQEmpty = 0, kSiteDqEmpty, kSiteMmaQFull, kSiteMmaFull, kSiteMmaPFull, kSiteMmaOFree,
+  kSiteSmSFull, kSiteSmVote, kSiteSmMax, kSiteSmFinal, kSiteSmPvRescale, kSiteSmLsum, kSiteSmL,
+  kSiteSmPvEpi, kSiteMmaFin
+};
+
+// Marks the CTA aborted; a wait that ran out (rather than saw the abort)
+// also records its site.
+__device__ __forceinline__ void set_abort(Ctrl& c, uint32_t* dev_err) {
+  *reinterpret_cast<volatile uint32_t*>(&c.abort) = 1u;
+  report(dev_err, QMLA_DEVERR_TIMEOUT);
+}
+__device__ __forceinline__ bool wait_ok(int r, uint32_t site, Ctrl& c, uint32_t* dev_err) {
+  if (r == 0) {
+    report(dev_err, QMLA_DEVERR_TIMEOUT | (0x100u << site));
+    *reinterpret_cast<volatile uint32_t*>(&c.abort) = 1u;
+  }
+  return r == 1;
+}
+// Warp-uniform bounded wait.
+__device__ __forceinline__ bool wwait(uint64_t* bar, uint32_t parity, Ctrl& c, uint32_t site,
+                                      uint32_t* dev_err) {
+  const bool ok = wait_ok(mbar_wait(bar, parity, kWaitNs, &c.abort), site, c, dev_err);
+  return __all_sync(0xffffffffu, ok);
+}
+// Barrier among the four softmax warps (one arrive per warp), bounded.
+__device__ __forceinline__ bool group_sync(uint64_t* bar, uint32_t& phase, Ctrl& c, uint32_t site,
+                                           uint32_t* dev_err) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
+  const bool ok = wwait(bar, phase & 1u, c, site, dev_err);
+  ++phase;
+  return ok;
+}
+
+// ------------------------------------------------------------- schedule
+struct Sched {
+  const int32_t* prefix;
+  int t0, t1, t, u, pu0, pu1;
+  int units;
+  __device__ void init(const int32_t* pf, int units_, int cta, int grid) {
+    prefix = pf;
+    units = units_;
+    const int T = pf[units];
+    t0 = static_cast<int>(static_cast<long long>(cta) * T / grid);
+    t1 = static_cast<int>(static_cast<long long>(cta + 1) * T / grid);
+    t = t0;
+    u = 0;
+    pu0 = pu1 = 0;
+    if (t0 >= t1) return;
+    int lo = 0, hi = units_;  // prefix[lo] <= t0 < prefix[hi]
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (pf[mid] <= t0) lo = mid; else hi = mid;
+    }
+    u = lo;
+    pu0 = pf[u];
+    pu1 = pf[u + 1];
+  }
+  __device__ bool valid() const { return t < t1; }
+  __device__ void next() {
+    ++t;
+    while (t < t1 && t >= pu1 && u + 1 < units) {
+      ++u;
+      pu0 = pu1;
+      pu1 = prefix[u + 1];
+    }
+  }
+};
+
+struct TileInfo {
+  int b, hg, j, ntok;
+  bool first, last;
+};
+__device__ __forceinline__ TileInfo tile_info(const Sched& s, const Params& p) {
+  TileInfo ti;
+  ti.b = s.u / p.n_hg;
+  ti.hg = s.u - ti.b * p.n_hg;
+  ti.j = s.t - s.pu0;
+  ti.ntok = min(kTileTokens, p.seq_lens[ti.b] - kTileTokens * ti.j);
+  ti.first = (s.t == s.t0) || (ti.j == 0);
+  ti.last = (s.t + 1 == s.t1) || (s.t + 1 == s.pu1);
+  return ti;
+}
+
+// -------------------------------------------------------- dequant warps
+// Packed data of one token row for one chunk, fetched ahead of use.
+struct Fetch {
+  uint4 a, b;
+  uint32_t sz;
+  bool ok;
+};
+
+template <int CB>
+__device__ __forceinline__ const uint8_t* row_block(const Params& p, const TileInfo& ti, int row,
+                                                    bool& valid) {
+  valid = row < ti.ntok;
+  if (!valid) return nullptr;
+  const int lb = 2 * ti.j + (row >> 6);
+  const int blk = p.table[static_cast<size_t>(ti.b) * p.max_blocks + lb];
+  if (blk < 0 || blk >= p.num_blocks) {
+    report(p.dev_err, QMLA_DEVERR_BAD_BLOCK);
+    valid = false;
+    return nullptr;
+  }
+  constexpr size_t kBlk = CB == 16 ? static_cast<size_t>(kBf16BlockBytes) : BlockLayout<CB == 16 ? 4 : CB>::kBytes;
+  return p.pool + static_cast<size_t>(blk) * kBlk;
+}
+
+template <int CB>
+__device__ __forceinline__ Fetch fetch_chunk(const uint8_t* blk, bool valid, int k, int slot) {
+  Fetch f;
+  f.ok = valid;
+  f.a = make_uint4(0, 0, 0, 0);
+  f.b = f.a;
+  f.sz = 0;
+  if (!valid) return f;
+  using L = BlockLayout<CB>;
+  const uint8_t* c = blk + L::code_off(k, slot);
+  f.a = ldg_nc_v4(c);
+  if (CB == 4 || k == 8) f.b = ldg_nc_v4(c + 16);
+  f.sz = ldg_nc_u32(blk + L::sz_off(k, slot));
+  return f;
+}
+
+// Unpacks one row (64 codes) of chunk k and stores RN_f16(s (q - z)) into the
+// swizzled chunk tile. The code nibbles / crumbs are placed into the mantissa
+// of 1024.0 (0x6400), giving 1024 + q exactly; subtracting 1024 + z is exact.
+template <int CB>
+__device__ __forceinline__ void store_row(uint32_t chunk_base, int row, const Fetch& f, bool int4) {
+  if (!f.ok) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) sts_v4(chunk_base + swz_off(row, i, 128), 0, 0, 0, 0);
+    return;
+  }
+  const __half2 sz = *reinterpret_cast<const __half2*>(&f.sz);
+  const __half2 s2 = __half2half2(__low2half(sz));
+  const __half2 zz2 = __half2half2(__hadd(__high2half(sz), __float2half_rn(1024.0f)));
+  const uint32_t ss = *reinterpret_cast<const uint32_t*>(&s2);
+  const uint32_t zz = *reinterpret_cast<const uint32_t*>(&zz2);
+  constexpr uint32_t K = 0x64646464u;
+  if (int4) {
+    const uint32_t w[8] = {f.a.x, f.a.y, f.a.z, f.a.w, f.b.x, f.b.y, f.b.z, f.b.w};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t lo = w[i] & 0x0F0F0F0Fu;          // e0 e2 e4 e6
+      const uint32_t hi = (w[i] >> 4) & 0x0F0F0F0Fu;   // e1 e3 e5 e7
+      sts_v4(chunk_base + swz_off(row, i, 128), dq2(__byte_perm(lo, K, 0x4140), zz, ss),
+             dq2(__byte_perm(hi, K, 0x4140), zz, ss), dq2(__byte_perm(lo, K, 0x4342), zz, ss),
+             dq2(__byte_perm(hi, K, 0x4342), zz, ss));
+    }
+  } else {
+    const uint32_t w[4] = {f.a.x, f.a.y, f.a.z, f.a.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const uint32_t c0 = w[i] & 0x03030303u;          // e0 e4 e8 e12
+      const uint32_t c1 = (w[i] >> 2) & 0x03030303u;   // e1 e5 e9 e13
+      const uint32_t c2 = (w[i] >> 4) & 0x03030303u;   // e2 e6 e10 e14
+      const uint32_t c3 = (w[i] >> 6) & 0x03030303u;   // e3 e7 e11 e15
+      sts_v4(chunk_base + swz_off(row, 2 * i, 128), dq2(__byte_perm(c0, K, 0x4140), zz, ss),
+             dq2(__byte_perm(c1, K, 0x4140), zz, ss), dq2(__byte_perm(c2, K, 0x4140), zz, ss),
+             dq2(__byte_perm(c3, K, 0x4140), zz, ss));
+      sts_v4(chunk_base + swz_off(row, 2 * i + 1, 128), dq2(__byte_perm(c0, K, 0x4342), zz, ss),
+             dq2(__byte_perm(c1, K, 0x4342), zz, ss), dq2(__byte_perm(c2, K, 0x4342), zz, ss),
+             dq2(__byte_perm(c3, K, 0x4342), zz, ss));
+    }
+  }
+}
+
+// BF16 comparison cache: the row is copied and rounded to fp16.
+__device__ __forceinline__ void store_row_bf16(uint32_t chunk_base, int row, const uint4 (&v)[8], bool ok) {
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    uint32_t o[4] = {0, 0, 0, 0};
+    if (ok) {
+      const uint32_t w[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) o[e] = pack_h2(bf16_lo(w[e]), bf16_hi(w[e]));
+    }
+    sts_v4(chunk_base + swz_off(row, i, 128), o[0], o[1], o[2], o[3]);
+  }
+}
+
+// Query tile: HG heads x 576 channels in fp16, K-major, 128-byte swizzle,
+// channels permuted within each 8-channel piece like the cache rows.
+template <int CB, int HG>
+__device__ void load_query(const Params& p, uint32_t qbase, int b, int h0, int tid, int nthreads) {
+  for (int idx = tid; idx < kNumChunks * HG * 8; idx += nthreads) {
+    const int i = idx & 7;
+    const int kh = idx >> 3;
+    const int h = kh % HG;
+    const int k = kh / HG;
+    uint4 raw = make_uint4(0, 0, 0, 0);
+    if (h0 + h < p.heads) {
+      const size_t bh = static_cast<size_t>(b) * p.heads + h0 + h;
+      const __nv_bfloat16* src = k < 8 ? p.q_lat + bh * kDc + k * 64 + i * 8 : p.q_pe + bh * kDr + i * 8;
+      raw = *reinterpret_cast<const uint4*>(src);
+    }
+    const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+    float f[8];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      f[2 * e] = bf16_lo(w[e]);
+      f[2 * e + 1] = bf16_hi(w[e]);
+    }
+    uint32_t o[4];
+    if (k < 8 || CB == 16) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) o[e] = pack_h2(f[Perm<CB>::at(2 * e)], f[Perm<CB>::at(2 * e + 1)]);
+    } else {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) o[e] = pack_h2(f[Perm<4>::at(2 * e)], f[Perm<4>::at(2 * e + 1)]);
+    }
+    sts_v4(qbase + k * HG * 128 + swz_off(h, i, 128), o[0], o[1], o[2], o[3]);
+  }
+}
+
+template <int CB, int HG>
+__device__ void dequant_role(const Params& p, Sched sc, uint32_t chunks, uint32_t qbase, Ctrl& ctl,
+                             int warp, int lane) {
+  const int row = (warp & 3) * 32 + lane;  // token row of the tile
+  const int par = warp >> 2;               // this warp handles chunks k = par, par+2, ...
+  const int slot = row & 63;
+  uint32_t it = 0, seg = 0;
+  Fetch f[5];
+  TileInfo ti;
+  bool ok = true;
+  if (sc.valid()) {
+    ti = tile_info(sc, p);
+    if constexpr (CB != 16) {
+      bool valid;
+      const uint8_t* blk = row_block<CB>(p, ti, row, valid);
+#pragma unroll
+      for (int kc = 0; kc < 5; ++kc) {
+        const int k = 2 * kc + par;
+        if (k < kNumChunks) f[kc] = fetch_chunk<CB>(blk, valid, k, slot);
+      }
+    }
+  }
+  while (ok && sc.valid()) {
+    if (ti.first) {
+      if (seg > 0 && !wwait(&ctl.q_empty, (seg - 1) & 1u, ctl, kSiteDqQEmpty, p.dev_err)) { ok = false; break; }
+      load_query<CB, HG>(p, qbase, ti.b, ti.hg * HG, warp * 32 + lane, kNumDqWarps * 32);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.q_full);
+    }
+    const uint8_t* blk16 = nullptr;
+    bool valid16 = false;
+    if constexpr (CB == 16) blk16 = row_block<CB>(p, ti, row, valid16);
+#pragma unroll
+    for (int kc = 0; kc < 5; ++kc) {
+      const int k = 2 * kc + par;
+      if (k >= kNumChunks) break;
+      if constexpr (CB == 16) {
+        uint4 v[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          v[i] = valid16 ? ldg_nc_v4(blk16 + slot * (kDqk * 2) + k * 128 + i * 16) : make_uint4(0, 0, 0, 0);
+        if (!wwait(&ctl.empty[k], (it & 1u) ^ 1u, ctl, kSiteDqEmpty, p.dev_err)) { ok = false; break; }
+        store_row_bf16(chunks + k * kChunkBytes, row, v, valid16);
+      } else {
+        if (!wwait(&ctl.empty[k], (it & 1u) ^ 1u, ctl, kSiteDqEmpty, p.dev_err)) { ok = false; break; }
+        store_row<CB>(chunks + k * kChunkBytes, row, f[kc], CB == 4 || k == 8);
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.full[k]);
+    }
+    if (!ok) break;
+    if (ti.last) ++seg;
+    ++it;
+    sc.next();
+    if (sc.valid()) {
+      ti = tile_info(sc, p);
+      if constexpr (CB != 16) {
+        bool valid;
+        const uint8_t* blk = row_block<CB>(p, ti, row, valid);
+#pragma unroll
+        for (int kc = 0; kc < 5; ++kc) {
+          const int k = 2 * kc + par;
+          if (k < kNumChunks) f[kc] = fetch_chunk<CB>(blk, valid, k, slot);
+        }
+      }
+    }
+  }
+  if (!ok) set_abort(ctl, p.dev_err);
+}
+
+// ------------------------------------------------------------ MMA warp
+// The whole warp walks the schedule and waits; lane 0 issues the MMAs and the
+// commits (a commit tracks the MMAs issued by the committing thread).
+template <int HG>
+__device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint32_t qbase, Ctrl& ctl,
+                         uint32_t tmem, int lane) {
+  constexpr uint32_t kIdQK = idesc_f16_f32(128, HG, false, false);
+  constexpr uint32_t kIdPV = idesc_f16_f32(128, HG, true, true);
+  constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
+  constexpr uint32_t kSboP = 8 * kRB;
+  const uint32_t ptile = chunks + 8 * kChunkBytes;
+  const uint32_t t_s = tmem + 4 * HG;
+  const bool leader = lane == 0;
+  uint32_t it = 0, seg = 0;
+  bool ok = true;
+  for (; ok && sc.valid(); sc.next()) {
+    const TileInfo ti = tile_info(sc, p);
+    if (ti.first && !(ok = wwait(&ctl.q_full, seg & 1u, ctl, kSiteMmaQFull, p.dev_err))) break;
+    // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576).
+    for (int k = 0; k < kNumChunks; ++k) {
+      if (!(ok = wwait(&ctl.full[k], it & 1u, ctl, kSiteMmaFull, p.dev_err))) break;
+      tc_fence_after();
+      if (leader) {
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          const uint64_t ad = smem_desc(chunks + k * kChunkBytes + kk * 32, 16, 1024, SWZ_128B);
+          const uint64_t bd = smem_desc(qbase + k * HG * 128 + kk * 32, 16, 1024, SWZ_128B);
+          umma_f16_ss(t_s, ad, bd, kIdQK, (k | kk) != 0 ? 1u : 0u);
+        }
+      }
+      __syncwarp();
+    }
+    if (!ok) break;
+    if (leader) {
+      umma_commit(&ctl.s_full);
+      if (ti.last) umma_commit(&ctl.q_empty);
+    }
+    __syncwarp();
+    if (!(ok = wwait(&ctl.p_full, it & 1u, ctl, kSiteMmaPFull, p.dev_err))) break;
+    if (ti.first && seg > 0 && !(ok = wwait(&ctl.o_free, (seg - 1) & 1u, ctl, kSiteMmaOFree, p.dev_err))) break;
+    tc_fence_after();
+    // O^T[c, h] += sum_t C_hat[t, c] P^T[t, h], 4 x 128 channels, K = 128 tokens.
+    if (leader) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint64_t ad = smem_desc(chunks + 2 * i * kChunkBytes + kk * 2048, kChunkBytes, 1024, SWZ_128B);
+          const uint64_t bd = smem_desc(ptile + kk * 2 * kSboP, 16 * kSboP, kSboP, swz_mode_for_row(kRB));
+          umma_f16_ss(tmem + i * HG, ad, bd, kIdPV, (ti.first && kk == 0) ? 0u : 1u);
+        }
+        umma_commit(&ctl.empty[2 * i]);
+        umma_commit(&ctl.empty[2 * i + 1]);
+      }
+      umma_commit(&ctl.empty[8]);
+      umma_commit(&ctl.pv_done);
+    }
+    __syncwarp();
+    ++it;
+    if (ti.last) ++seg;
+  }
+  if (!ok) set_abort(ctl, p.dev_err);
+  // Every MMA must have landed before TMEM is released, aborted or not.
+  if (leader) umma_commit(&ctl.fin);
+  __syncwarp();
+  wait_ok(mbar_wait(&ctl.fin, 0, kWaitNs, nullptr), kSiteMmaFin, ctl, p.dev_err);
+  __syncwarp();
+}
+
+// --------------------------------------------------------- softmax warps
+template <int CB, int HG>
+__device__ void softmax_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ctl, uint32_t tmem,
+                             int warp, int lane) {
+  const int q4 = warp & 3;
+  const int row = q4 * 32 + lane;
+  const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
+  const uint32_t t_s = tmem + 4 * HG + lane_off;
+  const uint32_t t_o = tmem + lane_off;
+  const uint32_t ptile = chunks + 8 * kChunkBytes;
+  constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
+  const float sl2 = p.scale_log2;
+  float lsum[HG];
+#pragma unroll
+  for (int h = 0; h < HG; ++h) lsum[h] = 0.0f;
+  uint32_t it = 0, gph[3] = {0, 0, 0};
+  int seg_j0 = 0;
+  bool ok = true;
+  for (; ok && sc.valid(); sc.next()) {
+    const TileInfo ti = tile_info(sc, p);
+    if (ti.first) seg_j0 = ti.j;
+    const bool valid = row < ti.ntok;
+    if (!(ok = wwait(&ctl.s_full, it & 1u, ctl, kSiteSmSFull, p.dev_err))) break;
+    tc_fence_after();
+    // Pass 1: does any score exceed the reference max by more than 2^8?
+    bool need = ti.first;
+    if (!ti.first) {
+#pragma unroll
+      for (int c = 0; c < HG / 16; ++c) {
+        uint32_t r[16];
+        tmem_ld16(t_s + c * 16, r);
+        tmem_ld_wait();
+#pragma unroll
+        for (int jj = 0; jj < 16; ++jj)
+          need |= valid && (__uint_as_float(r[jj]) * sl2 > ctl.m_ref[c * 16 + jj] + kRescaleLog2);
+      }
+    }
+    const uint32_t any = __any_sync(0xffffffffu, need);
+    uint32_t* vote = ctl.vote[it & 1u];
+    if (lane == 0) vote[q4] = any;
+    if (!(ok = group_sync(&ctl.grp[0], gph[0], ctl, kSiteSmVote, p.dev_err))) break;
+    if ((vote[0] | vote[1] | vote[2] | vote[3]) != 0u) {
+      // Tile max per head over the 128 tokens.
+#pragma unroll
+      for (int c = 0; c < HG / 16; ++c) {
+        uint32_t r[16];
+        tmem_ld16(t_s + c * 16, r);
+        tmem_ld_wait();
+#pragma unroll
+        for (int jj = 0; jj < 16; ++jj) {
+          const float x = valid ? __uint_as_float(r[jj]) * sl2 : -INFINITY;
+          const float mx = warp_max_f32(x);
+          if (lane == jj) ctl.red[q4][c * 16 + jj] = mx;
+        }
+      }
+      if (!(ok = group_sync(&ctl.grp[1], gph[1], ctl, kSiteSmMax, p.dev_err))) break;
+      if (row < HG) {
+        const float mt = fmaxf(fmaxf(ctl.red[0][row], ctl.red[1][row]), fmaxf(ctl.red[2][row], ctl.red[3][row]));
+        const float mo = ctl.m_ref[row];
+        const float mn = ti.first ? mt : fmaxf(mo, mt);
+        ctl.alpha[row] = ti.first ? 0.0f : exp2f(mo - mn);
+        ctl.m_ref[row] = mn;
+      }
+      if (!(ok = group_sync(&ctl.grp[2], gph[2], ctl, kSiteSmFinal, p.dev_err))) break;
+      if (ti.first) {
+#pragma unroll
+        for (int h = 0; h < HG; ++h) lsum[h] = 0.0f;
+      } else {
+        // O was accumulated against the old reference: wait for the previous
+        // PV to land, then scale every head's column by alpha.
+        if (!(ok = wwait(&ctl.pv_done, (it - 1) & 1u, ctl, kSiteSmPvRescale, p.dev_err))) break;
+        tc_fence_after();
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+#pragma unroll
+          for (int c = 0; c < HG / 16; ++c) {
+            uint32_t r[16];
+            tmem_ld16(t_o + i * HG + c * 16, r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int jj = 0; jj < 16; ++jj)
+              r[jj] = __float_as_uint(__uint_as_float(r[jj]) * ctl.alpha[c * 16 + jj]);
+            tmem_st16(t_o + i * HG + c * 16, r);
+          }
+        }
+        tmem_st_wait();
+#pragma unroll
+        for (int h = 0; h < HG; ++h) lsum[h] *= ctl.alpha[h];
+      }
+    }
+    // Pass 2: P^T[t, h] = 2^(S * scale * log2e - m_ref[h]) as fp16.
+#pragma unroll
+    for (int c = 0; c < HG / 16; ++c) {
+      uint32_t r[16];
+      tmem_ld16(t_s + c * 16, r);
+      tmem_ld_wait();
+      uint32_t pk[8];
+#pragma unroll
+      for (int jj = 0; jj < 16; jj += 2) {
+        const float p0 = valid ? exp2f(__uint_as_float(r[jj]) * sl2 - ctl.m_ref[c * 16 + jj]) : 0.0f;
+        const float p1 = valid ? exp2f(__uint_as_float(r[jj + 1]) * sl2 - ctl.m_ref[c * 16 + jj + 1]) : 0.0f;
+        const __half2 hp = __floats2half2_rn(p0, p1);
+        const float2 back = __half22float2(hp);
+        lsum[c * 16 + jj] += back.x;
+        lsum[c * 16 + jj + 1] += back.y;
+        pk[jj >> 1] = *reinterpret_cast<const uint32_t*>(&hp);
+      }
+      if constexpr (HG == 16) {
+        sts_v4(ptile + swz_off(row, 0, kRB), pk[0], pk[1], pk[2], pk[3]);
+        sts_v4(ptile + swz_off(row, 1, kRB), pk[4], pk[5], pk[6], pk[7]);
+      } else {
+        sts_v4(ptile + swz_off(row, 2 * c, kRB), pk[0], pk[1], pk[2], pk[3]);
+        sts_v4(ptile + swz_off(row, 2 * c + 1, kRB), pk[4], pk[5], pk[6], pk[7]);
+      }
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&ctl.p_full);
+
+    if (ti.last) {
+      // Segment end: l[h] = sum over the 128 token rows; then read O^T.
+#pragma unroll
+      for (int h = 0; h < HG; ++h) {
+        float v = lsum[h];
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+        if (lane == 0) ctl.red[q4][h] = v;
+      }
+      if (!(ok = group_sync(&ctl.grp[1], gph[1], ctl, kSiteSmLsum, p.dev_err))) break;
+      if (row < HG) ctl.alpha[row] = (ctl.red[0][row] + ctl.red[1][row]) + (ctl.red[2][row] + ctl.red[3][row]);
+      if (!(ok = group_sync(&ctl.grp[2], gph[2], ctl, kSiteSmL, p.dev_err))) break;
+      if (!(ok = wwait(&ctl.pv_done, it & 1u, ctl, kSiteSmPvEpi, p.dev_err))) break;
+      tc_fence_after();
+      const bool whole = (seg_j0 == 0) && (sc.t + 1 == sc.pu1);
+      const int h0 = ti.hg * HG;
+      const size_t pidx = static_cast<size_t>(blockIdx.x) + sc.u;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int P = i * 128 + row;  // position in the reconstructed row
+        const int ch = (P & ~7) + Perm<CB>::at(P & 7);
+#pragma unroll
+        for (int c = 0; c < HG / 16; ++c) {
+          uint32_t r[16];
+          tmem_ld16(t_o + i * HG + c * 16, r);
+          tmem_ld_wait();
+#pragma unroll
+          for (int jj = 0; jj < 16; ++jj) {
+            const int h = c * 16 + jj;
+            if (h0 + h < p.heads) {
+              const float v = __uint_as_float(r[jj]);
+              if (whole) {
+                p.out[(static_cast<size_t>(ti.b) * p.heads + h0 + h) * kDc + ch] = v / ctl.alpha[h];
+              } else {
+                p.part_o[(pidx * HG + h) * kDc + ch] = v;
+              }
+            }
+          }
+        }
+      }
+      if (row < HG && h0 + row < p.heads) {
+        if (whole) {
+          if (p.lse != nullptr)
+            p.lse[static_cast<size_t>(ti.b) * p.heads + h0 + row] = (ctl.m_ref[row] + log2f(ctl.alpha[row])) * kLn2;
+        } else {
+          p.part_ml[(pidx * HG + row) * 2 + 0] = ctl.m_ref[row];
+          p.part_ml[(pidx * HG + row) * 2 + 1] = ctl.alpha[row];
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.o_free);
+    }
+    ++it;
+  }
+  if (!ok) set_abort(ctl, p.dev_err);
+}
+
+template <int CB, int HG>
+__global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const uint32_t chunks = smem_u32(smem);
+  const uint32_t qbase = chunks + kNumChunks * kChunkBytes;
+  Ctrl& ctl = *reinterpret_cast<Ctrl*>(smem + kNumChunks * kChunkBytes + Cfg<HG>::kQBytes);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int k = 0; k < kNumChunks; ++k) {
+      mbar_init(&ctl.full[k], 4);
+      mbar_init(&ctl.empty[k], 1);
+    }
+    mbar_init(&ctl.s_full, 1);
+    mbar_init(&ctl.p_full, 4);
+    mbar_init(&ctl.pv_done, 1);
+    mbar_init(&ctl.o_free, 4);
+    mbar_init(&ctl.q_empty, 1);
+    mbar_init(&ctl.q_full, kNumDqWarps);
+    mbar_init(&ctl.fin, 1);
+    for (int i = 0; i < 3; ++i) mbar_init(&ctl.grp[i], 4);
+    ctl.abort = 0u;
+    fence_mbar_init();
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(&ctl.tmem_base, Cfg<HG>::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = ctl.tmem_base;
+
+  Sched sc;
+  sc.init(p.prefix, p.batch * p.n_hg, blockIdx.x, gridDim.x);
+  if (warp < kNumDqWarps) {
+    dequant_role<CB, HG>(p, sc, chunks, qbase, ctl, warp, lane);
+  } else if (warp < kMmaWarp) {
+    softmax_role<CB, HG>(p, sc, chunks, ctl, tmem, warp, lane);
+  } else {
+    mma_role<HG>(p, sc, chunks, qbase, ctl, tmem, lane);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc(tmem, Cfg<HG>::kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------ plan / combine
+__global__ void __launch_bounds__(1024) plan_kernel(const int32_t* __restrict__ seq_lens, int batch,
+                                                    int n_hg, int max_blocks, int32_t* __restrict__ prefix,
+                                                    uint32_t* dev_err) {
+  __shared__ int warp_sums[32];
+  __shared__ int carry;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nwarps = blockDim.x >> 5;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  for (int base = 0; base < batch; base += blockDim.x) {
+    const int b = base + threadIdx.x;
+    int tiles = 0;
+    if (b < batch) {
+      int len = seq_lens[b];
+      if (len < 0 || len > max_blocks * kBlockTokens) {
+        report(dev_err, QMLA_DEVERR_BAD_POSITION);
+        len = 0;
+      }
+      tiles = (len + kTileTokens - 1) / kTileTokens;
+    }
+    const int v = tiles * n_hg;
+    int x = v;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, x, off);
+      if (lane >= off) x += y;
+    }
+    if (lane == 31) warp_sums[warp] = x;
+    __syncthreads();
+    if (warp == 0) {
+      int s = lane < nwarps ? warp_sums[lane] : 0;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, s, off);
+        if (lane >= off) s += y;
+      }
+      warp_sums[lane] = s;
+    }
+    __syncthreads();
+    const int excl = carry + (warp > 0 ? warp_sums[warp - 1] : 0) + x - v;
+    if (b < batch) {
+      for (int hg = 0; hg < n_hg; ++hg) prefix[b * n_hg + hg] = excl + hg * tiles;
+    }
+    __syncthreads();
+    if (threadIdx.x == blockDim.x - 1) carry = excl + v;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) prefix[batch * n_hg] = carry;
+}
+
+// First tile of CTA c's range, and the CTA whose range holds tile t.
+__device__ __forceinline__ int cta_start(int c, int T, int grid) {
+  return static_cast<int>(static_cast<long long>(c) * T / grid);
+}
+__device__ __forceinline__ int cta_of(int t, int T, int grid) {
+  return static_cast<int>((static_cast<long long>(t + 1) * grid - 1) / T);
+}
+
+template <int HG>
+__global__ void __launch_bounds__(256) combine_kernel(const Params p) {
+  const int u = blockIdx.x;
+  const int units = p.batch * p.n_hg;
+  const int b = u / p.n_hg;
+  const int h0 = (u - b * p.n_hg) * HG;
+  const int nh = min(HG, p.heads - h0);
+  const int P0 = p.prefix[u], P1 = p.prefix[u + 1], T = p.prefix[units];
+  float* out = p.out + (static_cast<size_t>(b) * p.heads + h0) * kDc;
+  if (P0 == P1) {
+    for (int idx = threadIdx.x; idx < nh * kDc; idx += blockDim.x) out[idx] = 0.0f;
+    if (p.lse != nullptr && threadIdx.x < nh) p.lse[static_cast<size_t>(b) * p.heads + h0 + threadIdx.x] = -INFINITY;
+    return;
+  }
+  const int c0 = cta_of(P0, T, p.grid), c1 = cta_of(P1 - 1, T, p.grid);
+  if (c0 == c1) return;  // one CTA covered the whole unit and wrote the result
+  for (int idx = threadIdx.x; idx < nh * (kDc / 4); idx += blockDim.x) {
+    const int h = idx / (kDc / 4);
+    const int q = idx - h * (kDc / 4);
+    // CTAs between c0 and c1 with an empty range wrote no partial.
+    float M = -INFINITY;
+    for (int c = c0; c <= c1; ++c) {
+      if (cta_start(c, T, p.grid) == cta_start(c + 1, T, p.grid)) continue;
+      M = fmaxf(M, p.part_ml[((static_cast<size_t>(c) + u) * HG + h) * 2]);
+    }
+    float s = 0.0f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c = c0; c <= c1; ++c) {
+      if (cta_start(c, T, p.grid) == cta_start(c + 1, T, p.grid)) continue;
+      const size_t pi = (static_cast<size_t>(c) + u) * HG + h;
+      const float w = exp2f(p.part_ml[pi * 2] - M);
+      s += w * p.part_ml[pi * 2 + 1];
+      const float4 o = reinterpret_cast<const float4*>(p.part_o + pi * kDc)[q];
+      acc.x += w * o.x;
+      acc.y += w * o.y;
+      acc.z += w * o.z;
+      acc.w += w * o.w;
+    }
+    const float inv = 1.0f / s;
+    reinterpret_cast<float4*>(out + static_cast<size_t>(h) * kDc)[q] =
+        make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+    if (q == 0 && p.lse != nullptr) p.lse[static_cast<size_t>(b) * p.heads + h0 + h] = (M + log2f(s)) * kLn2;
+  }
+}
+
+template <int CB, int HG>
+cudaError_t launch_impl(const Params& prm, cudaStream_t stream) {
+  static int configured_device = -1;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (configured_device != dev) {
+    e = cudaFuncSetAttribute(decode_main<CB, HG>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<HG>::kSmem);
+    if (e != cudaSuccess) return e;
+    configured_device = dev;
+  }
+  decode_main<CB, HG><<<prm.grid, kThreads, Cfg<HG>::kSmem, stream>>>(prm);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  combine_kernel<HG><<<prm.batch * prm.n_hg, 256, 0, stream>>>(prm);
+  return cudaGetLastError();
+}
+
+template <int CB>
+cudaError_t launch_hg(int hg, const Params& prm, cudaStream_t stream) {
+  if (hg == 16) return launch_impl<CB, 16>(prm, stream);
+  if (hg == 32) return launch_impl<CB, 32>(prm, stream);
+  return launch_impl<CB, 64>(prm, stream);
+}
+
+}  // namespace
+
+int head_group_size(int heads) { return heads <= 16 ? 16 : (heads <= 32 ? 32 : 64); }
+
+DecodeWorkspace decode_workspace_layout(int batch, int heads, int grid) {
+  const int hg = head_group_size(heads);
+  const size_t units = static_cast<size_t>(batch) * ((heads + hg - 1) / hg);
+  auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
+  DecodeWorkspace w;
+  w.prefix_off = 0;
+  w.part_o_off = up((units + 1) * sizeof(int32_t));
+  const size_t nparts = static_cast<size_t>(grid) + units;
+  w.part_ml_off = w.part_o_off + up(nparts * hg * kDc * sizeof(float));
+  w.total = w.part_ml_off + up(nparts * hg * 2 * sizeof(float));
+  return w;
+}
+
+cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
+  const int hg = head_group_size(a.heads);
+  const DecodeWorkspace w = decode_workspace_layout(a.batch, a.heads, a.grid);
+  uint8_t* ws = static_cast<uint8_t*>(a.workspace);
+  Params prm;
+  prm.pool = static_cast<const uint8_t*>(a.pool);
+  prm.num_blocks = a.num_blocks;
+  prm.q_lat = reinterpret_cast<const __nv_bfloat16*>(a.q_latent);
+  prm.q_pe = reinterpret_cast<const __nv_bfloat16*>(a.q_pe);
+  prm.batch = a.batch;
+  prm.heads = a.heads;
+  prm.n_hg = (a.heads + hg - 1) / hg;
+  prm.table = a.table;
+  prm.max_blocks = a.max_blocks;
+  prm.seq_lens = a.seq_lens;
+  prm.scale_log2 = a.softmax_scale * 1.4426950408889634f;
+  prm.out = a.out;
+  prm.lse = a.lse;
+  prm.prefix = reinterpret_cast<const int32_t*>(ws + w.prefix_off);
+  prm.prefix_w = reinterpret_cast<int32_t*>(ws + w.prefix_off);
+  prm.part_o = reinterpret_cast<float*>(ws + w.part_o_off);
+  prm.part_ml = reinterpret_cast<float*>(ws + w.part_ml_off);
+  prm.dev_err = a.dev_err;
+  prm.grid = a.grid;
+  plan_kernel<<<1, 1024, 0, stream>>>(a.seq_lens, a.batch, prm.n_hg, a.max_blocks, prm.prefix_w, a.dev_err);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  if (a.cache_kind == 4) return launch_hg<4>(hg, prm, stream);
+  if (a.cache_kind == 2) return launch_hg<2>(hg, prm, stream);
+  return launch_hg<16>(hg, prm, stream);
+}
+
+}  // namespace qmla

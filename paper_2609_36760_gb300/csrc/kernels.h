@@ -1,0 +1,47 @@
+// Internal launchers shared by the C ABI (api.cu) and the kernel files.
+#pragma once
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace qmla {
+
+cudaError_t launch_quant_append(void* pool, int c_bits, int num_blocks, const uint16_t* latent,
+                                const uint16_t* k_pe, const int32_t* seq_ids,
+                                const int32_t* positions, int n, const int32_t* table, int num_seqs,
+                                int max_blocks, uint32_t* dev_err, cudaStream_t stream);
+
+cudaError_t launch_bf16_append(void* pool, int num_blocks, const uint16_t* latent,
+                               const uint16_t* k_pe, const int32_t* seq_ids,
+                               const int32_t* positions, int n, const int32_t* table, int num_seqs,
+                               int max_blocks, uint32_t* dev_err, cudaStream_t stream);
+
+// Heads handled by one CTA (the N of every MMA): 16, 32 or 64.
+int head_group_size(int heads);
+
+// Workspace carve-up of the decode path for `grid` CTAs.
+struct DecodeWorkspace {
+  size_t prefix_off, part_o_off, part_ml_off, total;
+};
+DecodeWorkspace decode_workspace_layout(int batch, int heads, int grid);
+
+struct DecodeArgs {
+  const void* pool;
+  int cache_kind;  // 4 or 2: packed content bits; 16: BF16 cache
+  int num_blocks;
+  const uint16_t* q_latent;
+  const uint16_t* q_pe;
+  int batch, heads;
+  const int32_t* table;
+  int max_blocks;
+  const int32_t* seq_lens;
+  float softmax_scale;
+  float* out;
+  float* lse;
+  void* workspace;
+  uint32_t* dev_err;
+  int grid;  // CTAs of the main kernel (one per SM)
+};
+cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
+
+}  // namespace qmla

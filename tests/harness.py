@@ -1,0 +1,148 @@
+"""Test harness: drives the CUDA library and the CPU oracle on the same seeded inputs.
+
+The oracle sees only the generator's bf16 inputs (never anything the GPU
+produced); the GPU sees the same bytes through the library's C ABI.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import torch
+
+import paper_2609_36760_gb300 as Q
+from oracle import attention as OA
+from oracle import layout as OL
+from oracle import quantizer as OQ
+from workloads import synthetic as W
+
+TAU = 1.0 / math.sqrt(192.0)
+POISON = 0xAB
+
+
+def rel_l2(a, b) -> float:
+    a = np.asarray(a, np.float64)
+    b = np.asarray(b, np.float64)
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
+
+
+class Case:
+    """A workload materialised on the GPU (packed or BF16 cache) plus its inputs on the host."""
+
+    def __init__(self, w: W.Workload, bf16_cache: bool = False, device: str = "cuda"):
+        self.w = w
+        self.bf16 = bf16_cache
+        self.dev = device
+        self.prefill = W.seq_lengths(w)
+        self.final = W.final_lengths(w)
+        table, nblocks = W.block_table(w)
+        self.table = table
+        self.nblocks = nblocks
+        self.gains = W.channel_gains(w)
+        bb = Q.bf16_block_bytes() if bf16_cache else Q.block_bytes(w.c_bits)
+        self.pool = torch.full((nblocks, bb), POISON, dtype=torch.uint8, device=device)
+        self.table_d = table.to(device)
+        self.dev_err = torch.zeros(1, dtype=torch.int32, device=device)
+        self._tok = {}
+
+    # host-side inputs, cached per sequence (bf16 tensors up to the final length)
+    def tokens(self, b: int):
+        if b not in self._tok:
+            n = self.final[b]
+            self._tok[b] = (W.latent_for_seq(self.w, b, n, self.gains), W.kpe_for_seq(self.w, b, n))
+        return self._tok[b]
+
+    def append(self, lat: torch.Tensor, kpe: torch.Tensor, seq_ids, positions) -> None:
+        lat_d = lat.contiguous().to(self.dev)
+        kpe_d = kpe.contiguous().to(self.dev)
+        sid = None if seq_ids is None else torch.as_tensor(seq_ids, dtype=torch.int32).to(self.dev)
+        pos = torch.as_tensor(positions, dtype=torch.int32).to(self.dev)
+        if self.bf16:
+            Q.bf16_append(self.pool, lat_d, kpe_d, sid, pos, self.table_d, self.dev_err)
+        else:
+            Q.quant_append(self.pool, self.w.c_bits, lat_d, kpe_d, sid, pos, self.table_d, self.dev_err)
+
+    def prefill_all(self, chunk_tokens: int = 1 << 20) -> None:
+        """Writes tokens [0, prefill_b) of every sequence."""
+        lats, kps, sids, poss = [], [], [], []
+        pending = 0
+        for b in range(self.w.batch):
+            n = self.prefill[b]
+            if n == 0:
+                continue
+            lat, kp = self.tokens(b)
+            lats.append(lat[:n]); kps.append(kp[:n])
+            sids.append(torch.full((n,), b, dtype=torch.int32)); poss.append(torch.arange(n, dtype=torch.int32))
+            pending += n
+            if pending >= chunk_tokens:
+                self.append(torch.cat(lats), torch.cat(kps), torch.cat(sids), torch.cat(poss))
+                lats, kps, sids, poss, pending = [], [], [], [], 0
+        if pending:
+            self.append(torch.cat(lats), torch.cat(kps), torch.cat(sids), torch.cat(poss))
+
+    def lengths_at(self, step: int) -> list[int]:
+        return [n + self.w.append * (step + 1) for n in self.prefill]
+
+    def append_step(self, step: int) -> None:
+        """Writes the ``append`` tokens of every sequence for decode step ``step``."""
+        if self.w.append == 0:
+            return
+        lats, kps, sids, poss = [], [], [], []
+        for b in range(self.w.batch):
+            lat, kp = self.tokens(b)
+            a0 = self.prefill[b] + self.w.append * step
+            for k in range(self.w.append):
+                lats.append(lat[a0 + k:a0 + k + 1]); kps.append(kp[a0 + k:a0 + k + 1])
+                sids.append(b); poss.append(a0 + k)
+        self.append(torch.cat(lats), torch.cat(kps), sids, poss)
+
+    def decode(self, step: int, lens: list[int] | None = None, queries=None):
+        ql, qp = queries if queries is not None else W.queries(self.w, step)
+        lens = self.lengths_at(step) if lens is None else lens
+        B, H = self.w.batch, self.w.heads
+        out = torch.full((B, H, 512), float("nan"), dtype=torch.float32, device=self.dev)
+        lse = torch.full((B, H), float("nan"), dtype=torch.float32, device=self.dev)
+        ws = Q.workspace_for(B, H, self.dev)
+        ws.fill_(0x7F)
+        sl = torch.tensor(lens, dtype=torch.int32, device=self.dev)
+        ql_d, qp_d = ql.contiguous().to(self.dev), qp.contiguous().to(self.dev)
+        if self.bf16:
+            Q.mla_decode_bf16cache(self.pool, ql_d, qp_d, self.table_d, sl, TAU, out, lse, ws, self.dev_err)
+        else:
+            Q.mla_decode(self.pool, self.w.c_bits, ql_d, qp_d, self.table_d, sl, TAU, out, lse, ws, self.dev_err)
+        torch.cuda.synchronize()
+        return out.cpu().numpy(), lse.cpu().numpy()
+
+    def dev_error(self) -> int:
+        return Q.read_dev_err(self.dev_err)
+
+    # ---------------------------------------------------------------- oracle side
+    def oracle_cache(self, b: int, L: int, fp16_tiles: bool = False):
+        lat, kp = self.tokens(b)
+        latf = lat[:L].double().numpy()
+        kpf = kp[:L].double().numpy()
+        if self.bf16:
+            return latf, kpf
+        q, s, z = OL.quantize_tokens(latf, kpf, self.w.c_bits)
+        if fp16_tiles:
+            x = OQ.dequantize_fp16(q.reshape(L, 9, 64), s, z).astype(np.float64).reshape(L, 576)
+            return x[:, :512], x[:, 512:]
+        return OA.dequantize_tokens(q, s, z)
+
+    def oracle_decode(self, b: int, L: int, step: int = 0, heads=None, fp16_tiles: bool = False, queries=None):
+        ql, qp = queries if queries is not None else W.queries(self.w, step)
+        C, K = self.oracle_cache(b, L, fp16_tiles)
+        hs = slice(None) if heads is None else heads
+        return OA.attend(ql[b, hs].double().numpy(), qp[b, hs].double().numpy(), C, K, TAU)
+
+    def oracle_pool_blocks(self, seqs, upto: list[int]):
+        """Oracle-written bytes of the blocks owned by ``seqs`` (tokens [0, upto[b]))."""
+        bb = OL.block_bytes(self.w.c_bits)
+        pool = np.full((self.nblocks, bb), POISON, np.uint8)
+        for b in seqs:
+            lat, kp = self.tokens(b)
+            n = upto[b]
+            OL.write_tokens(pool, self.w.c_bits, lat[:n].double().numpy(), kp[:n].double().numpy(),
+                            np.full(n, b), np.arange(n), self.table.numpy())
+        blocks = sorted({int(x) for b in seqs for x in self.table[b].tolist() if x >= 0})
+        return blocks, pool[blocks]

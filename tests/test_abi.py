@@ -1,0 +1,73 @@
+"""The C-ABI library builds, loads, exports every symbol include/qmla.h declares,
+and validates arguments on the host (no GPU needed for any of this)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "qmla.h")
+
+
+@pytest.fixture(scope="module")
+def libqmla():
+    import paper_2609_36760_gb300 as Q
+    from paper_2609_36760_gb300 import build
+    if not os.path.exists(Q.library_path()):
+        build.build()
+    return Q.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(qmla_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ["qmla_quant_append", "qmla_mla_decode", "qmla_mla_decode_bf16cache", "qmla_block_bytes",
+                     "qmla_decode_workspace_bytes", "qmla_read_dev_err", "qmla_bf16_append"]:
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(libqmla):
+    for name in declared_functions():
+        assert hasattr(libqmla, name), name
+
+
+def test_pure_host_queries(libqmla):
+    assert libqmla.qmla_block_bytes(4) == 20736
+    assert libqmla.qmla_block_bytes(2) == 12544
+    assert libqmla.qmla_block_bytes(3) == 0 and libqmla.qmla_block_bytes(8) == 0
+    assert libqmla.qmla_bf16_block_bytes() == 73728
+    assert libqmla.qmla_status_string(0) == b"ok"
+    assert libqmla.qmla_status_string(3) == b"workspace too small"
+
+
+def test_invalid_arguments_are_rejected_before_any_launch(libqmla):
+    L = libqmla
+    fake = ctypes.c_void_p(0x10000)  # never dereferenced: validation fails first
+    # bad bit width
+    assert L.qmla_quant_append(fake, 3, 4, fake, fake, None, fake, 1, fake, 1, 1, None, None) == 1
+    # null positions
+    assert L.qmla_quant_append(fake, 4, 4, fake, fake, None, None, 1, fake, 1, 1, None, None) == 1
+    # misaligned pool
+    assert L.qmla_quant_append(ctypes.c_void_p(0x10001), 4, 4, fake, fake, None, fake, 1, fake, 1, 1, None, None) == 1
+    # n == 0 is a no-op that touches nothing
+    assert L.qmla_quant_append(None, 4, 4, None, None, None, None, 0, None, 1, 1, None, None) == 0
+    # decode: heads out of range, null output, bad scale, bad bits
+    args = [fake, 4, 4, fake, fake, 1, 129, fake, 1, fake, 0.1, fake, None, fake, 1 << 30, None, None]
+    assert L.qmla_mla_decode(*args) == 1
+    args[6] = 16
+    args[11] = None
+    assert L.qmla_mla_decode(*args) == 1
+    args[11] = fake
+    args[10] = -1.0
+    assert L.qmla_mla_decode(*args) == 1
+    args[10] = 0.1
+    args[1] = 8
+    assert L.qmla_mla_decode(*args) == 1
+    assert L.qmla_decode_workspace_bytes(0, 16) == 0
+    assert L.qmla_decode_workspace_bytes(1, 0) == 0

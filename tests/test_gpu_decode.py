@@ -1,0 +1,202 @@
+"""Parity of qmla_mla_decode (and its BF16-cache variant) with the fp64 oracle.
+
+Bar (on every workload): max |out - oracle| <= 2e-3 and
+||out - oracle|| / ||oracle|| <= 1e-3, with the oracle attending over the exact
+dequantised cache s (q - z). Edge cases whose outputs are dominated by a few
+large tokens are additionally checked against the oracle evaluated on the
+fp16-rounded reconstruction RN_f16(s (q - z)) that the kernel's tiles hold,
+where the only remaining differences are the fp16 rounding of the softmax
+weights (relative 2^-11 each, so at most ~5e-4 of the largest |value|) and fp32
+accumulation: there the bar is max-abs <= 1e-3 * max(1, max|ref|) and
+rel-L2 <= 1e-3. Very short contexts (a handful of tokens) are checked only
+that way: their output is a few reconstructed tokens, whose fp16 rounding alone
+can exceed 2e-3 on the x8 outlier channels.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_36760_gb300 as Q
+from harness import TAU, Case, rel_l2
+from workloads import synthetic as W
+
+pytestmark = pytest.mark.gpu
+
+MAX_ABS = 2e-3
+REL_L2 = 1e-3
+LSE_ABS = 1e-3
+
+
+def check(case: Case, step: int, seqs, got_out, got_lse, max_abs=MAX_ABS, rel=REL_L2, fp16_tiles=False,
+          queries=None):
+    lens = case.lengths_at(step)
+    outs, refs, lses, rlses = [], [], [], []
+    for b in seqs:
+        ref, rlse = case.oracle_decode(b, lens[b], step, fp16_tiles=fp16_tiles, queries=queries)
+        outs.append(got_out[b]); refs.append(ref); lses.append(got_lse[b]); rlses.append(rlse)
+    o, r = np.stack(outs), np.stack(refs)
+    assert np.isfinite(o).all()
+    err = np.max(np.abs(o - r))
+    rl = rel_l2(o, r)
+    assert err <= max_abs, f"max-abs {err:.3e}"
+    assert rl <= rel, f"rel-L2 {rl:.3e}"
+    assert np.max(np.abs(np.stack(lses) - np.stack(rlses))) <= LSE_ABS
+    return err, rl
+
+
+def check_tile(case: Case, step: int, seqs, got_out, got_lse, queries=None):
+    """Against the oracle on the fp16-rounded reconstruction (tile-exact)."""
+    lens = case.lengths_at(step)
+    for b in seqs:
+        ref, rlse = case.oracle_decode(b, lens[b], step, fp16_tiles=True, queries=queries)
+        if lens[b] == 0:
+            continue
+        scale = max(1.0, float(np.abs(ref).max()))
+        assert np.max(np.abs(got_out[b] - ref)) <= 1e-3 * scale, f"seq {b}"
+        assert rel_l2(got_out[b], ref) <= 1e-3, f"seq {b}"
+        assert np.max(np.abs(got_lse[b] - rlse)) <= LSE_ABS
+
+
+def run_case(w, bf16=False):
+    c = Case(w, bf16_cache=bf16)
+    c.prefill_all()
+    c.append_step(0)
+    out, lse = c.decode(0)
+    assert c.dev_error() == 0
+    return c, out, lse
+
+
+def test_tiny_workload_full():
+    c, out, lse = run_case(W.WORKLOADS["tiny_b1_h16_l256_int4"])
+    check(c, 0, [0], out, lse)
+
+
+@pytest.mark.parametrize("bits", [4, 2])
+@pytest.mark.parametrize("heads", [1, 16, 20, 64, 100, 128])
+def test_shapes_and_ragged_tails(bits, heads):
+    lengths = (1, 2, 63, 64, 65, 127, 128, 129, 300, 1000)
+    w = W.small_workload("s", batch=len(lengths), heads=heads, lengths=lengths, c_bits=bits, seed=21 + heads,
+                         latent_dist="gauss_gain_outlier" if bits == 4 else "t4_gain")
+    c, out, lse = run_case(w)
+    check_tile(c, 0, range(w.batch), out, lse)
+    check(c, 0, [b for b in range(w.batch) if c.prefill[b] >= 256], out, lse)
+
+
+def test_bf16_cache_variant():
+    w = W.small_workload("b", batch=5, heads=64, lengths=(1, 64, 129, 700, 2000), seed=31)
+    c, out, lse = run_case(w, bf16=True)
+    check_tile(c, 0, range(w.batch), out, lse)
+    check(c, 0, [3, 4], out, lse)
+    w2 = W.small_workload("b2", batch=3, heads=128, lengths=(5, 4097, 200), seed=32)
+    c2, out2, lse2 = run_case(w2, bf16=True)
+    check_tile(c2, 0, range(w2.batch), out2, lse2)
+    check(c2, 0, [1], out2, lse2)
+
+
+def test_split_units_and_combine():
+    # Far more tiles than SMs: every (sequence, head group) is split across
+    # several CTAs and merged by the combine kernel.
+    w = W.small_workload("split", batch=3, heads=128, lengths=(20000, 9000, 130), seed=41)
+    c, out, lse = run_case(w)
+    check(c, 0, range(w.batch), out, lse)
+
+
+def test_same_answer_at_any_split():
+    # The same sequence decoded alone (few splits) and next to long neighbours
+    # (many splits) agrees to fp32 accumulation-order noise.
+    w_alone = W.small_workload("a", batch=1, heads=64, lengths=(5000,), seed=51)
+    c1, out1, _ = run_case(w_alone)
+    w_many = W.small_workload("a", batch=4, heads=64, lengths=(5000, 60000, 60000, 60000), seed=51)
+    c2, out2, _ = run_case(w_many)
+    assert np.max(np.abs(out1[0] - out2[0])) <= 1e-4
+
+
+def test_empty_and_single_token_sequences():
+    w = W.small_workload("e", batch=4, heads=16, lengths=(0, 1, 0, 65), seed=61)
+    c = Case(w)
+    c.prefill_all()
+    out, lse = c.decode(0, lens=[0, 1, 0, 65])
+    assert np.all(out[0] == 0) and np.all(out[2] == 0)
+    assert np.all(np.isneginf(lse[0])) and np.all(np.isneginf(lse[2]))
+    # one token: every head's output is that token's reconstruction RN_f16(s (q - z))
+    Cf, _ = c.oracle_cache(1, 1, fp16_tiles=True)
+    assert np.array_equal(out[1], np.repeat(Cf[:1].astype(np.float32), 16, axis=0))
+    check_tile(c, 0, [3], out, lse)
+    assert c.dev_error() == 0
+
+
+def test_rescale_path_growing_scores():
+    # Scores that grow along the sequence force the reference max to move by far
+    # more than 2^8 between tiles, exercising the O rescaling.
+    w = W.small_workload("r", batch=2, heads=64, lengths=(1500, 700), seed=71)
+    c = Case(w)
+    for b in range(w.batch):
+        lat, kp = c.tokens(b)
+        ramp = torch.linspace(0.2, 3.0, lat.shape[0], dtype=torch.float64)[:, None]
+        c._tok[b] = ((lat.double() * ramp).to(torch.bfloat16), kp)
+    c.prefill_all()
+    ql, qp = W.queries(w, 0)
+    ql = (ql.double() * 40.0).to(torch.bfloat16)
+    out, lse = c.decode(0, queries=(ql, qp))
+    assert c.dev_error() == 0
+    assert np.isfinite(out).all()
+    # Largest score gap along the sequence, in log2 units, must exceed the threshold.
+    S = []
+    for b in range(w.batch):
+        C, K = c.oracle_cache(b, c.prefill[b])
+        s = TAU * (ql[b].double().numpy() @ C.T + qp[b].double().numpy() @ K.T) / math.log(2)
+        S.append(s[:, -128:].max() - s[:, :128].max())
+    assert max(S) > 16
+    lens = c.prefill
+    for b in range(w.batch):
+        ref, rlse = c.oracle_decode(b, lens[b], 0, fp16_tiles=True, queries=(ql, qp))
+        scale = np.abs(ref).max()
+        assert np.max(np.abs(out[b] - ref)) <= 2e-3 * scale
+        assert rel_l2(out[b], ref) <= 1e-3
+        assert np.max(np.abs(lse[b] - rlse)) <= 1e-3 * max(1.0, np.abs(rlse).max())
+
+
+def test_bad_block_id_flags_error_and_stays_finite():
+    w = W.small_workload("bad", batch=2, heads=16, lengths=(200, 200), seed=81)
+    c = Case(w)
+    c.prefill_all()
+    t = c.table.clone()
+    t[1, 1] = 1 << 20
+    c.table_d = t.cuda()
+    out, lse = c.decode(0)
+    assert c.dev_error() & Q.DEVERR_BAD_BLOCK
+    assert np.isfinite(out).all()
+    # sequence 0 is unaffected
+    check_tile(c, 0, [0], out, lse)
+
+
+def test_seq_len_beyond_table_flags_error():
+    w = W.small_workload("over", batch=2, heads=16, lengths=(64, 64), seed=82)
+    c = Case(w)
+    c.prefill_all()
+    out, lse = c.decode(0, lens=[64, 64 * 50])
+    assert c.dev_error() & Q.DEVERR_BAD_POSITION
+    assert np.all(out[1] == 0) and np.all(np.isneginf(lse[1]))
+
+
+@pytest.mark.parametrize("name", ["dsv3_b64_h128_l4096_int4", "int2_b32_h128_l32768", "long_b4_h64_l128k"])
+def test_full_size_workloads(name):
+    w = W.WORKLOADS[name]
+    c, out, lse = run_case(w)
+    seqs = sorted({0, w.batch // 2, w.batch - 1})
+    check(c, 0, seqs, out, lse)
+
+
+def test_serving_mix_256_steps():
+    w = W.WORKLOADS["serve_b128_h16_mix"]
+    c = Case(w)
+    c.prefill_all()
+    seqs = [0, 77, 127]
+    for step in range(w.steps):
+        c.append_step(step)
+        if step in (0, 1, 128, w.steps - 1):
+            out, lse = c.decode(step)
+            check(c, step, seqs, out, lse)
+    assert c.dev_error() == 0

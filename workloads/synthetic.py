@@ -104,9 +104,11 @@ def latent_for_seq(w: Workload, b: int, n_tokens: int, gains: torch.Tensor | Non
         gains = channel_gains(w)
     if w.latent_dist == "gauss_gain_outlier":
         x = torch.randn(n_tokens, D_C, generator=g, dtype=torch.float64)
-    else:  # Student-t with 4 degrees of freedom: N / sqrt(chi2_4 / 4)
+    else:  # Student-t with 4 degrees of freedom: N / sqrt(chi2_4 / 4),
+        # chi2_4 = -2 ln(U1 U2) (a sum of two exponentials with mean 2)
         z = torch.randn(n_tokens, D_C, generator=g, dtype=torch.float64)
-        chi = torch.randn(n_tokens, D_C, 4, generator=g, dtype=torch.float64).pow(2).sum(-1)
+        u = 1.0 - torch.rand(2, n_tokens, D_C, generator=g, dtype=torch.float64)
+        chi = -2.0 * (torch.log(u[0]) + torch.log(u[1]))
         x = z / torch.sqrt(chi / 4.0)
     return (x * gains).to(torch.bfloat16)
 
