@@ -1,0 +1,470 @@
+#!/usr/bin/env python3
+"""Benchmark of the low-bit MLA decode hot path on GB300.
+
+One step = qmla_quant_append of one new token per sequence followed by
+qmla_mla_decode over every cached token (plan + main + combine kernels), on
+the DeepSeek-V3-shaped workload (64 sequences x 128 heads, 4096 cached tokens
+plus the appended one, INT4 content + INT4 RoPE key) unless --workload says
+otherwise. The metric is KV-tokens/s: tokens attended per step / step time.
+
+Contract: `python bench.py --gpus N --steps K --warmup W` prints one JSON line
+(rank 0). With N > 1 (torchrun) every rank decodes its own copy of the
+workload (independent sequences, no collective on the data path): weak
+scaling, max time over ranks. `--impl reference` times the CPU oracle instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+from workloads import synthetic as W  # noqa: E402
+
+METRIC = "low-bit MLA decode KV-tokens/s and µs/step on 1 GB300; % of roofline"
+UNIT = "KV-tokens/s"
+DEFAULT_WORKLOAD = "dsv3_b64_h128_l4096_int4"
+TAU = 1.0 / math.sqrt(192.0)
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["native", "reference"], default="native")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(W.WORKLOADS))
+    ap.add_argument("--bf16-cache", action="store_true", help="decode the BF16 comparison cache instead")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": float(d["hbm_gbs"]), "bf16_tflops": float(d["bf16_tflops"])}, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def workload_cost(w: W.Workload, lens: list[int], bf16: bool):
+    """Algorithmic FLOPs and HBM bytes of one decode launch (see the design notes)."""
+    tokens = sum(lens)
+    flops = 2.0 * w.heads * (576 + 512) * tokens
+    per_tok = 1152 if bf16 else (324 if w.c_bits == 4 else 196)
+    nbytes = tokens * per_tok + w.batch * w.heads * (576 * 2 + 512 * 4 + 4)
+    return flops, nbytes
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled while the timed loop runs."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.idx = device_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.12)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, smax, reasons = [], [], set()
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, v in zip(["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"], f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def profile_traffic(kernel_file_hash: str):
+    """DRAM bytes per main-kernel launch from the committed ncu summary, if it
+    was taken on the current kernel source; otherwise None."""
+    p = os.path.join(ROOT, "profiles", "decode_main_traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    if d.get("decode_cu_sha256") != kernel_file_hash:
+        return None
+    return d
+
+
+def decode_cu_hash() -> str:
+    with open(os.path.join(ROOT, "paper_2609_36760_gb300", "csrc", "decode.cu"), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+# ------------------------------------------------------------------ native
+class Workspace:
+    """GPU state of one workload: pool, block table, per-step inputs."""
+
+    def __init__(self, w: W.Workload, bf16: bool, dev: torch.device, nsteps: int):
+        import paper_2609_36760_gb300 as Q
+        self.Q = Q
+        self.w, self.bf16, self.dev = w, bf16, dev
+        self.prefill = W.seq_lengths(w)
+        table, nblocks = W.block_table(w)
+        self.table = table.to(dev)
+        bb = Q.bf16_block_bytes() if bf16 else Q.block_bytes(w.c_bits)
+        self.pool = torch.zeros((nblocks, bb), dtype=torch.uint8, device=dev)
+        self.err = torch.zeros(1, dtype=torch.int32, device=dev)
+        gains = W.channel_gains(w)
+        self.nsteps = max(1, min(nsteps, w.steps))
+        self.step_in = [dict(lat=[], kp=[], pos=[]) for _ in range(self.nsteps)]
+        # Prefill through the library, one sequence at a time (bounded host memory).
+        for b in range(w.batch):
+            n_all = self.prefill[b] + w.append * self.nsteps
+            lat = W.latent_for_seq(w, b, n_all, gains)
+            kp = W.kpe_for_seq(w, b, n_all)
+            n = self.prefill[b]
+            self._append(lat[:n].to(dev), kp[:n].to(dev), torch.full((n,), b, dtype=torch.int32, device=dev),
+                         torch.arange(n, dtype=torch.int32, device=dev))
+            for s in range(self.nsteps):
+                for k in range(w.append):
+                    p = n + w.append * s + k
+                    self.step_in[s]["lat"].append(lat[p:p + 1])
+                    self.step_in[s]["kp"].append(kp[p:p + 1])
+                    self.step_in[s]["pos"].append(p)
+        torch.cuda.synchronize(dev)
+        self.steps = []
+        for s in range(self.nsteps):
+            si = self.step_in[s]
+            ql, qp = W.queries(w, s)
+            lens = [n + w.append * (s + 1) for n in self.prefill]
+            host = {
+                "lat": torch.cat(si["lat"]) if si["lat"] else torch.zeros(0, 512, dtype=torch.bfloat16),
+                "kp": torch.cat(si["kp"]) if si["kp"] else torch.zeros(0, 64, dtype=torch.bfloat16),
+                "sid": torch.tensor([b for b in range(w.batch) for _ in range(w.append)], dtype=torch.int32),
+                "pos": torch.tensor(si["pos"], dtype=torch.int32),
+                "ql": ql.contiguous(), "qp": qp.contiguous(),
+                "lens": torch.tensor(lens, dtype=torch.int32),
+            }
+            self.steps.append({"host": host, "dev": {k: v.to(dev) for k, v in host.items()}, "lens": lens})
+        self.out = torch.empty((w.batch, w.heads, 512), dtype=torch.float32, device=dev)
+        self.lse = torch.empty((w.batch, w.heads), dtype=torch.float32, device=dev)
+        self.ws = Q.workspace_for(w.batch, w.heads, dev)
+
+    def _append(self, lat, kp, sid, pos):
+        if lat.shape[0] == 0:
+            return
+        if self.bf16:
+            self.Q.bf16_append(self.pool, lat, kp, sid, pos, self.table, self.err)
+        else:
+            self.Q.quant_append(self.pool, self.w.c_bits, lat, kp, sid, pos, self.table, self.err)
+
+    def step(self, s: int, d: dict | None = None, out=None, lse=None):
+        d = d if d is not None else self.steps[s % self.nsteps]["dev"]
+        out = self.out if out is None else out
+        lse = self.lse if lse is None else lse
+        self._append(d["lat"], d["kp"], d["sid"], d["pos"])
+        if self.bf16:
+            self.Q.mla_decode_bf16cache(self.pool, d["ql"], d["qp"], self.table, d["lens"], TAU, out, lse, self.ws,
+                                        self.err)
+        else:
+            self.Q.mla_decode(self.pool, self.w.c_bits, d["ql"], d["qp"], self.table, d["lens"], TAU, out, lse,
+                              self.ws, self.err)
+
+    def launches_per_step(self) -> int:
+        return (1 if self.w.append > 0 else 0) + 3
+
+
+def run_native(args, ws_world: int, rank: int, local: int):
+    import paper_2609_36760_gb300 as Q
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    Q.lib()
+    dist = None
+    if ws_world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    w = W.WORKLOADS[args.workload]
+    K, Wm = args.steps, args.warmup
+    state = Workspace(w, args.bf16_cache, dev, K + Wm)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # larger than the 126 MB L2
+    stream = torch.cuda.current_stream(dev)
+
+    # warm-up (untimed)
+    for i in range(Wm):
+        flush.zero_()
+        state.step(i)
+    torch.cuda.synchronize(dev)
+    if Q.read_dev_err(state.err) != 0:
+        raise RuntimeError(f"device error word {Q.read_dev_err(state.err):#x} after warm-up")
+
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
+    for e in ev:
+        for x in e:
+            x.record(stream)
+    torch.cuda.synchronize(dev)
+    clocks = ClockSampler(local)
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    clocks.start()
+    time.sleep(0.15)
+    t_wall0 = time.perf_counter()
+    for i in range(K):
+        e0, e1, e_m0, e_m1 = ev[i]
+        flush.zero_()
+        Q.set_profile_events(e_m0, e_m1)
+        e0.record(stream)
+        state.step(Wm + i)
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    t_wall = time.perf_counter() - t_wall0
+    Q.set_profile_events(None, None)
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    clk = clocks.stop()
+    err = Q.read_dev_err(state.err)
+    if err != 0:
+        raise RuntimeError(f"device error word {err:#x} in the timed loop")
+
+    step_ms = [ev[i][0].elapsed_time(ev[i][1]) for i in range(K)]
+    main_ms = [ev[i][2].elapsed_time(ev[i][3]) for i in range(K)]
+    ms_step = sum(step_ms) / K
+    ms_main = sum(main_ms) / K
+    if dist is not None:
+        t = torch.tensor([ms_step], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_step_max = float(t.item())
+    else:
+        ms_step_max = ms_step
+
+    lens_all = [state.steps[(Wm + i) % state.nsteps]["lens"] for i in range(K)]
+    tok_per_step = sum(sum(l) for l in lens_all) / K
+    value = ws_world * tok_per_step / (ms_step_max * 1e-3)
+
+    # roofline of the main decode kernel
+    peaks, peak_src = load_peaks()
+    flops, nbytes = workload_cost(w, lens_all[0], args.bf16_cache)
+    t_tc = flops / (peaks["bf16_tflops"] * 1e12)
+    t_hbm = nbytes / (peaks["hbm_gbs"] * 1e9)
+    tensor_bound = t_tc >= t_hbm
+    if tensor_bound:
+        achieved = flops / (ms_main * 1e-3) / 1e12
+        roof = {"bound": "tensor", "achieved": round(achieved, 2), "peak": peaks["bf16_tflops"], "unit": "TFLOP/s"}
+    else:
+        achieved = nbytes / (ms_main * 1e-3) / 1e9
+        roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s"}
+    roof["frac"] = round(achieved / roof["peak"], 4)
+    roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
+    prof = profile_traffic(decode_cu_hash())
+    roof["traffic"] = (prof["dram_bytes_per_launch"] if prof and prof.get("workload") == args.workload
+                       and bool(prof.get("bf16_cache")) == bool(args.bf16_cache) else None)
+    roof["kernel"] = "decode_main"
+    roof["kernel_us"] = round(ms_main * 1e3, 2)
+    roof["algorithmic_flops"] = flops
+    roof["algorithmic_bytes"] = nbytes
+    roof["roofline_us"] = round(max(t_tc, t_hbm) * 1e6, 2)
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(state, K=min(K, 200), flush=flush, dev=dev, tokens=tok_per_step, n_world=ws_world, dist=dist)
+
+    res = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": ws_world, "steps": K, "warmup": Wm,
+        "ms_per_step": round(ms_step_max, 5), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f16", "data": "synthetic (seeded generators, workloads/synthetic.py)",
+        "config": {"workload": w.name, "batch_per_gpu": w.batch, "heads": w.heads, "c_bits": w.c_bits,
+                   "pe_bits": 4, "cache": "bf16" if args.bf16_cache else f"int{w.c_bits}/int4 packed",
+                   "kv_tokens_per_step_per_gpu": tok_per_step, "l2": "flushed (256 MB write) before every timed step",
+                   "parallelism": f"replicas x{ws_world} (independent sequences)"},
+        "us_per_step": round(ms_step_max * 1e3, 2),
+        "roofline": roof,
+        "gpu_launches": state.launches_per_step() * K,
+        "clocks": clk,
+        "e2e": e2e,
+        "wall_s_timed_loop": round(t_wall, 3),
+    }
+    if rank == 0 and ws_world == 1 and not args.no_cpu_baseline:
+        res["cpu_baseline"] = cpu_baseline(w, args.bf16_cache, budget_s=15.0)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(res), flush=True)
+
+
+def run_e2e(state: Workspace, K: int, flush, dev, tokens: float, n_world: int, dist):
+    """Same metric through the public API with the step's inputs in pinned host
+    memory: H2D copies of the appended tokens, queries and lengths, and the D2H
+    read of out and lse, all inside the timed region."""
+    stream = torch.cuda.current_stream(dev)
+    hs = []
+    for s in range(state.nsteps):
+        h = {k: v.pin_memory() for k, v in state.steps[s]["host"].items()}
+        d = {k: torch.empty_like(v, device=dev) for k, v in h.items()}
+        hs.append((h, d))
+    out_h = torch.empty(state.out.shape, dtype=torch.float32).pin_memory()
+    lse_h = torch.empty(state.lse.shape, dtype=torch.float32).pin_memory()
+    h2d = sum(v.numel() * v.element_size() for v in hs[0][0].values())
+    d2h = out_h.numel() * 4 + lse_h.numel() * 4
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    for i in range(K + 3):
+        h, d = hs[i % state.nsteps]
+        flush.zero_()
+        if i >= 3:
+            evs[i - 3][0].record(stream)
+        for k in h:
+            d[k].copy_(h[k], non_blocking=True)
+        state.step(i, d)
+        out_h.copy_(state.out, non_blocking=True)
+        lse_h.copy_(state.lse, non_blocking=True)
+        if i >= 3:
+            evs[i - 3][1].record(stream)
+        stream.synchronize()
+    ms = sum(a.elapsed_time(b) for a, b in evs) / K
+    if dist is not None:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return {"value": round(n_world * tokens / (ms * 1e-3), 1), "unit": UNIT, "ms_per_step": round(ms, 5),
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": K}
+
+
+# ------------------------------------------------------------------ oracle
+def oracle_step_sample(w: W.Workload, bf16: bool, budget_s: float, max_seqs: int | None = None):
+    """Times the CPU oracle on one decode step (append of the step's tokens,
+    read-back and dequantisation of each sequence's cache, fp64 attention) for
+    as many sequences as fit in `budget_s`. Returns (tokens, seconds, nseq)."""
+    import numpy as np
+    from oracle import attention as OA
+    from oracle import layout as OL
+
+    prefill = W.seq_lengths(w)
+    gains = W.channel_gains(w)
+    ql, qp = W.queries(w, 0)
+    tot_tok, tot_s, nseq = 0, 0.0, 0
+    limit = w.batch if max_seqs is None else min(max_seqs, w.batch)
+    for b in range(limit):
+        n = prefill[b]
+        L = n + w.append
+        lat = W.latent_for_seq(w, b, L, gains).double().numpy()
+        kp = W.kpe_for_seq(w, b, L).double().numpy()
+        row = np.arange((L + 63) // 64, dtype=np.int64)
+        if not bf16:
+            pool = np.zeros((len(row), OL.block_bytes(w.c_bits)), np.uint8)
+            OL.write_tokens(pool, w.c_bits, lat[:n], kp[:n], np.zeros(n, np.int64), np.arange(n), row[None, :])
+        t0 = time.perf_counter()
+        if bf16:
+            C, K = lat, kp
+        else:
+            if w.append:
+                OL.write_tokens(pool, w.c_bits, lat[n:L], kp[n:L], np.zeros(L - n, np.int64), np.arange(n, L),
+                                row[None, :])
+            q, s, z = OL.read_sequence(pool, w.c_bits, row, L)
+            C, K = OA.dequantize_tokens(q, s, z)
+        OA.attend(ql[b].double().numpy(), qp[b].double().numpy(), C, K, TAU)
+        tot_s += time.perf_counter() - t0
+        tot_tok += L
+        nseq += 1
+        if tot_s >= budget_s:
+            break
+    return tot_tok, tot_s, nseq
+
+
+def cpu_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(w: W.Workload, bf16: bool, budget_s: float):
+    tok, sec, nseq = oracle_step_sample(w, bf16, budget_s)
+    return {"value": round(tok / sec, 1), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+            "sample": f"{nseq} of {w.batch} sequences of one decode step ({tok} KV tokens, "
+                      f"{w.heads} heads): append + cache read-back + dequantisation + fp64 attention, "
+                      f"numpy with BLAS threads = host cores; {sec:.2f} s"}
+
+
+def run_reference(args, ws_world: int, rank: int):
+    if rank != 0:
+        return
+    w = W.WORKLOADS[args.workload]
+    # Each step is a bounded sample: at most 4 sequences of the step.
+    steps = []
+    for i in range(args.warmup + args.steps):
+        tok, sec, nseq = oracle_step_sample(w, args.bf16_cache, budget_s=1e9, max_seqs=min(4, w.batch))
+        if i >= args.warmup:
+            steps.append((tok, sec))
+    tok = sum(t for t, _ in steps)
+    sec = sum(s for _, s in steps)
+    value = tok / sec
+    res = {"impl": "reference", "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": ws_world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * sec / len(steps), 3),
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic (seeded generators, workloads/synthetic.py)",
+           "config": {"workload": w.name, "batch_per_gpu": w.batch, "heads": w.heads, "c_bits": w.c_bits,
+                      "pe_bits": 4, "sample_per_step": f"{min(4, w.batch)} sequences"},
+           "cpu_baseline": {"value": round(value, 1), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                            "sample": f"{min(4, w.batch)} of {w.batch} sequences per step, {len(steps)} steps"},
+           "e2e": {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(res), flush=True)
+
+
+def main():
+    args = parse()
+    ws_world, rank, local = dist_env()
+    if args.impl == "reference":
+        run_reference(args, ws_world, rank)
+        return
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA device (the native path has no CPU fallback)")
+    run_native(args, ws_world, rank, local)
+
+
+if __name__ == "__main__":
+    main()

@@ -158,6 +158,13 @@ int qmla_mla_decode_bf16cache(const void* pool_dev, int num_blocks, const uint16
                               float* lse_dev, void* workspace_dev, size_t workspace_bytes,
                               uint32_t* dev_err_dev, qmla_stream_t stream);
 
+/* Measurement hook. While set (per host thread), every qmla_mla_decode* call
+ * records the caller-owned CUDA events `before_main` and `after_main`
+ * (cudaEvent_t, may be NULL) on its stream immediately before and after the
+ * main decode kernel, so the caller can time that kernel alone with
+ * cudaEventElapsedTime. Pass NULL, NULL to stop. Always returns QMLA_OK. */
+int qmla_set_profile_events(void* before_main, void* after_main);
+
 /* Copies the device error word to *host_out after synchronising `stream`. */
 int qmla_read_dev_err(const uint32_t* dev_err_dev, uint32_t* host_out, qmla_stream_t stream);
 

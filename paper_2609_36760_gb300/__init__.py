@@ -63,6 +63,7 @@ def lib():
     L.qmla_last_cuda_error.argtypes, L.qmla_last_cuda_error.restype = [], i32
     L.qmla_status_string.argtypes, L.qmla_status_string.restype = [i32], ctypes.c_char_p
     L.qmla_num_sms.argtypes, L.qmla_num_sms.restype = [], i32
+    L.qmla_set_profile_events.argtypes, L.qmla_set_profile_events.restype = [vp, vp], i32
     _lib = L
     return L
 
@@ -145,6 +146,14 @@ def mla_decode_bf16cache(pool: torch.Tensor, q_latent: torch.Tensor, q_pe: torch
                                          workspace.numel() * workspace.element_size(), _ptr(dev_err),
                                          _stream(stream))
     _check("qmla_mla_decode_bf16cache", st)
+
+
+def set_profile_events(before_main: torch.cuda.Event | None, after_main: torch.cuda.Event | None) -> None:
+    """qmla_set_profile_events: record these (already recorded once, so that
+    they exist) events around the main decode kernel of later decode calls."""
+    h0 = ctypes.c_void_p(before_main.cuda_event) if before_main is not None else None
+    h1 = ctypes.c_void_p(after_main.cuda_event) if after_main is not None else None
+    lib().qmla_set_profile_events(h0, h1)
 
 
 def read_dev_err(dev_err: torch.Tensor, stream=None) -> int:

@@ -11,6 +11,8 @@
 namespace {
 
 thread_local int g_last_cuda_error = 0;
+thread_local cudaEvent_t g_ev_before_main = nullptr;
+thread_local cudaEvent_t g_ev_after_main = nullptr;
 
 int cuda_fail(cudaError_t e) {
   g_last_cuda_error = static_cast<int>(e);
@@ -93,6 +95,8 @@ int decode_common(const void* pool, int kind, int num_blocks, const uint16_t* q_
   a.workspace = workspace;
   a.dev_err = dev_err;
   a.grid = di.sms;
+  a.ev_before_main = g_ev_before_main;
+  a.ev_after_main = g_ev_after_main;
   cudaError_t e = qmla::launch_decode(a, reinterpret_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
 }
@@ -175,7 +179,22 @@ int qmla_read_dev_err(const uint32_t* dev_err_dev, uint32_t* host_out, qmla_stre
   return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
 }
 
+int qmla_set_profile_events(void* before_main, void* after_main) {
+  g_ev_before_main = static_cast<cudaEvent_t>(before_main);
+  g_ev_after_main = static_cast<cudaEvent_t>(after_main);
+  return QMLA_OK;
+}
+
 int qmla_last_cuda_error(void) { return g_last_cuda_error; }
+
+#ifdef QMLA_TRACE_BUILD
+// Trace builds only (libqmla_trace.so): device buffer that receives the
+// decode kernel's per-CTA event timeline; NULL disables.
+int qmla_trace_set(void* buf_dev) {
+  cudaError_t e = qmla::set_trace_buffer(buf_dev);
+  return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
+}
+#endif
 
 const char* qmla_status_string(int status) {
   switch (status) {

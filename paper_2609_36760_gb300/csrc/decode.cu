@@ -2,9 +2,12 @@
 // "cache update and tile reuse" and "global attention normalization").
 //
 // Three kernels run per decode call:
-//   plan_kernel    per-sequence tile counts -> prefix over (sequence, head group)
-//                  units; the flattened tile list is cut into one equal range per
-//                  SM ("metadata construction", App. F.1).
+//   prep_kernel    block 0: per-sequence tile counts -> prefix over (sequence,
+//                  head group) units; the flattened tile list is cut into one
+//                  equal range per SM ("metadata construction", App. F.1).
+//                  Other blocks: query preparation, bf16 -> fp16 in the exact
+//                  swizzled shared-memory image the MMA reads, one image per
+//                  unit, later copied into each CTA by the bulk-copy engine.
 //   decode_main    one persistent CTA per SM walks its tile range. A tile is 128
 //                  cached tokens (two 64-token blocks) for one head group of HG
 //                  heads. Per tile:
@@ -31,6 +34,8 @@
 //                  m = max m_j, l = sum e^(m_j - m) l_j, O = sum e^(m_j - m) o_j / l.
 #include <cuda_runtime.h>
 
+#include <cstddef>
+
 #include "common.cuh"
 #include "kernels.h"
 #include "ptx.cuh"
@@ -49,6 +54,23 @@ constexpr uint64_t kWaitNs = 2000000000ull;      // bound of every on-chip wait 
 constexpr float kRescaleLog2 = 8.0f;             // rescale O only above 2^8 growth
 constexpr float kLn2 = 0.6931471805599453f;
 
+// Optional per-CTA timeline (clock64 at pipeline events), compiled in only
+// for trace builds (-DQMLA_TRACE_BUILD); see qmla_trace_set in api.cu.
+#ifdef QMLA_TRACE_BUILD
+constexpr int kTraceCtas = 8, kTraceEvents = 96, kTraceTiles = 32;
+__device__ unsigned long long* g_trace = nullptr;
+#define QMLA_TRACE(ev, tile)                                                                     \
+  do {                                                                                           \
+    if (g_trace != nullptr && blockIdx.x < kTraceCtas && (tile) < kTraceTiles)                   \
+      g_trace[(static_cast<size_t>(blockIdx.x) * kTraceEvents + (ev)) * kTraceTiles + (tile)] = \
+          clock64();                                                                             \
+  } while (0)
+#else
+#define QMLA_TRACE(ev, tile) \
+  do {                       \
+  } while (0)
+#endif
+
 struct Params {
   const uint8_t* pool;
   int num_blocks;
@@ -65,27 +87,32 @@ struct Params {
   int32_t* prefix_w;
   float* part_o;   // [(grid + units)][HG][512]
   float* part_ml;  // [(grid + units)][HG][2]
+  uint8_t* qimg;   // [units][9][HG][128 B]: swizzled fp16 query tiles
   uint32_t* dev_err;
   int grid;
 };
 
 struct __align__(16) Ctrl {
-  uint64_t full[kNumChunks];
-  uint64_t empty[kNumChunks];
-  uint64_t s_full, p_full, pv_done, o_free, q_empty, q_full, fin;
+  // tile_full: every chunk of the tile is written (one arrive per dequant warp).
+  // pv_done: the tile's PV has completed, so every chunk slot is free again.
+  uint64_t tile_full, s_full, p_full, pv_done, o_free, q_full, fin;
   uint64_t grp[3];
   uint32_t tmem_base;
   uint32_t abort;
   uint32_t vote[2][4];
-  float m_ref[64];
-  float alpha[64];
-  float red[4][64];
+  alignas(16) float m_ref[64];  // read as float4
+  alignas(16) float alpha[64];
+  alignas(16) float red[4][64];
 };
+static_assert(offsetof(Ctrl, m_ref) % 16 == 0 && offsetof(Ctrl, alpha) % 16 == 0, "float4 access alignment");
+static_assert(sizeof(Ctrl) % 16 == 0, "Ctrl size");
 
 template <int HG>
 struct Cfg {
   static constexpr int kQBytes = kNumChunks * HG * 128;
+  // O^T (4 HG columns), S^T (HG), row sums of P (HG), rounded up to a power of 2.
   static constexpr uint32_t kTmemCols = HG == 64 ? 512 : (HG == 32 ? 256 : 128);
+  static_assert(6 * HG <= static_cast<int>(kTmemCols), "TMEM columns");
   static constexpr int kSmem = 1024 + kNumChunks * kChunkBytes + kQBytes + (int)sizeof(Ctrl);
   static constexpr uint32_t kPRowBytes = 2 * HG;  // P^T tile row (one token, HG fp16)
 };
@@ -149,7 +176,7 @@ __device__ __forceinline__ float warp_max_f32(float v) {
 
 // Wait sites, reported in bits 8.. of the error word when a wait runs out.
 enum WaitSite : uint32_t {
-  kSiteDqQEmpty = 0, kSiteDqEmpty, kSiteMmaQFull, kSiteMmaFull, kSiteMmaPFull, kSiteMmaOFree,
+  kSiteDqEmpty = 0, kSiteMmaQFull, kSiteMmaFull, kSiteMmaPFull, kSiteMmaOFree,
   kSiteSmSFull, kSiteSmVote, kSiteSmMax, kSiteSmFinal, kSiteSmPvRescale, kSiteSmLsum, kSiteSmL,
   kSiteSmPvEpi, kSiteMmaFin
 };
@@ -167,11 +194,20 @@ __device__ __forceinline__ bool wait_ok(int r, uint32_t site, Ctrl& c, uint32_t*
   }
   return r == 1;
 }
-// Warp-uniform bounded wait.
+// Warp-uniform bounded wait: lane 0 polls (mbarrier polls share the
+// shared-memory pipe with the tensor core's operand reads, so one poller per
+// warp keeps them cheap), then every lane acquires the completed phase once.
 __device__ __forceinline__ bool wwait(uint64_t* bar, uint32_t parity, Ctrl& c, uint32_t site,
                                       uint32_t* dev_err) {
-  const bool ok = wait_ok(mbar_wait(bar, parity, kWaitNs, &c.abort), site, c, dev_err);
-  return __all_sync(0xffffffffu, ok);
+  int r = 1;
+  if ((threadIdx.x & 31) == 0) r = mbar_wait(bar, parity, kWaitNs, &c.abort);
+  r = __shfl_sync(0xffffffffu, r, 0);
+  if (r == 1) {
+    (void)mbar_test(bar, parity);
+  } else if ((threadIdx.x & 31) == 0) {
+    wait_ok(r, site, c, dev_err);
+  }
+  return r == 1;
 }
 // Barrier among the four softmax warps (one arrive per warp), bounded.
 __device__ __forceinline__ bool group_sync(uint64_t* bar, uint32_t& phase, Ctrl& c, uint32_t site,
@@ -331,47 +367,48 @@ __device__ __forceinline__ void store_row_bf16(uint32_t chunk_base, int row, con
   }
 }
 
-// Query tile: HG heads x 576 channels in fp16, K-major, 128-byte swizzle,
-// channels permuted within each 8-channel piece like the cache rows.
+// Query image of one unit: HG heads x 576 channels in fp16 laid out exactly as
+// the K-major, 128-byte-swizzled shared-memory operand ([chunk][head][128 B]),
+// channels permuted within each 8-channel piece like the cache rows. Piece
+// (k, h, i) is 8 channels of chunk k, head h. bf16 -> fp16 is exact for
+// magnitudes in [2^-14, 65504].
 template <int CB, int HG>
-__device__ void load_query(const Params& p, uint32_t qbase, int b, int h0, int tid, int nthreads) {
-  for (int idx = tid; idx < kNumChunks * HG * 8; idx += nthreads) {
-    const int i = idx & 7;
-    const int kh = idx >> 3;
-    const int h = kh % HG;
-    const int k = kh / HG;
-    uint4 raw = make_uint4(0, 0, 0, 0);
-    if (h0 + h < p.heads) {
-      const size_t bh = static_cast<size_t>(b) * p.heads + h0 + h;
-      const __nv_bfloat16* src = k < 8 ? p.q_lat + bh * kDc + k * 64 + i * 8 : p.q_pe + bh * kDr + i * 8;
-      raw = *reinterpret_cast<const uint4*>(src);
-    }
-    const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
-    float f[8];
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      f[2 * e] = bf16_lo(w[e]);
-      f[2 * e + 1] = bf16_hi(w[e]);
-    }
-    uint32_t o[4];
-    if (k < 8 || CB == 16) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) o[e] = pack_h2(f[Perm<CB>::at(2 * e)], f[Perm<CB>::at(2 * e + 1)]);
-    } else {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) o[e] = pack_h2(f[Perm<4>::at(2 * e)], f[Perm<4>::at(2 * e + 1)]);
-    }
-    sts_v4(qbase + k * HG * 128 + swz_off(h, i, 128), o[0], o[1], o[2], o[3]);
+__device__ __forceinline__ void query_piece(const Params& p, uint8_t* img, int b, int h0, int idx) {
+  const int i = idx & 7;
+  const int kh = idx >> 3;
+  const int h = kh % HG;
+  const int k = kh / HG;
+  uint4 raw = make_uint4(0, 0, 0, 0);
+  if (h0 + h < p.heads) {
+    const size_t bh = static_cast<size_t>(b) * p.heads + h0 + h;
+    const __nv_bfloat16* src = k < 8 ? p.q_lat + bh * kDc + k * 64 + i * 8 : p.q_pe + bh * kDr + i * 8;
+    raw = *reinterpret_cast<const uint4*>(src);
   }
+  const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+  float f[8];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    f[2 * e] = bf16_lo(w[e]);
+    f[2 * e + 1] = bf16_hi(w[e]);
+  }
+  uint4 o;
+  uint32_t* ov = reinterpret_cast<uint32_t*>(&o);
+  if (k < 8 || CB == 16) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) ov[e] = pack_h2(f[Perm<CB>::at(2 * e)], f[Perm<CB>::at(2 * e + 1)]);
+  } else {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) ov[e] = pack_h2(f[Perm<4>::at(2 * e)], f[Perm<4>::at(2 * e + 1)]);
+  }
+  *reinterpret_cast<uint4*>(img + k * HG * 128 + swz_off(h, i, 128)) = o;
 }
 
 template <int CB, int HG>
-__device__ void dequant_role(const Params& p, Sched sc, uint32_t chunks, uint32_t qbase, Ctrl& ctl,
-                             int warp, int lane) {
+__device__ void dequant_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ctl, int warp, int lane) {
   const int row = (warp & 3) * 32 + lane;  // token row of the tile
   const int par = warp >> 2;               // this warp handles chunks k = par, par+2, ...
   const int slot = row & 63;
-  uint32_t it = 0, seg = 0;
+  uint32_t it = 0;
   Fetch f[5];
   TileInfo ti;
   bool ok = true;
@@ -388,37 +425,52 @@ __device__ void dequant_role(const Params& p, Sched sc, uint32_t chunks, uint32_
     }
   }
   while (ok && sc.valid()) {
-    if (ti.first) {
-      if (seg > 0 && !wwait(&ctl.q_empty, (seg - 1) & 1u, ctl, kSiteDqQEmpty, p.dev_err)) { ok = false; break; }
-      load_query<CB, HG>(p, qbase, ti.b, ti.hg * HG, warp * 32 + lane, kNumDqWarps * 32);
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl.q_full);
+    // Phased schedule: the tile is written while the tensor pipe is idle
+    // (after the previous tile's PV), because generic shared-memory stores
+    // are starved while the tensor core streams its operands.
+    if (!wwait(&ctl.pv_done, (it & 1u) ^ 1u, ctl, kSiteDqEmpty, p.dev_err)) {
+      ok = false;
+      break;
     }
-    const uint8_t* blk16 = nullptr;
-    bool valid16 = false;
-    if constexpr (CB == 16) blk16 = row_block<CB>(p, ti, row, valid16);
+    if (lane == 0 && warp == 0) QMLA_TRACE(0, it);
+    if (lane == 0) QMLA_TRACE(40 + warp, it);
+    if constexpr (CB == 16) {
+      bool valid16 = false;
+      const uint8_t* blk16 = row_block<CB>(p, ti, row, valid16);
+      uint4 v[8];
 #pragma unroll
-    for (int kc = 0; kc < 5; ++kc) {
-      const int k = 2 * kc + par;
-      if (k >= kNumChunks) break;
-      if constexpr (CB == 16) {
-        uint4 v[8];
+      for (int i = 0; i < 8; ++i)
+        v[i] = valid16 ? ldg_nc_v4(blk16 + slot * (kDqk * 2) + par * 128 + i * 16) : make_uint4(0, 0, 0, 0);
 #pragma unroll
-        for (int i = 0; i < 8; ++i)
-          v[i] = valid16 ? ldg_nc_v4(blk16 + slot * (kDqk * 2) + k * 128 + i * 16) : make_uint4(0, 0, 0, 0);
-        if (!wwait(&ctl.empty[k], (it & 1u) ^ 1u, ctl, kSiteDqEmpty, p.dev_err)) { ok = false; break; }
-        store_row_bf16(chunks + k * kChunkBytes, row, v, valid16);
-      } else {
-        if (!wwait(&ctl.empty[k], (it & 1u) ^ 1u, ctl, kSiteDqEmpty, p.dev_err)) { ok = false; break; }
-        store_row<CB>(chunks + k * kChunkBytes, row, f[kc], CB == 4 || k == 8);
+      for (int kc = 0; kc < 5; ++kc) {
+        const int k = 2 * kc + par;
+        if (k >= kNumChunks) break;
+        uint4 cur[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) cur[i] = v[i];
+        if (k + 2 < kNumChunks) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            v[i] = valid16 ? ldg_nc_v4(blk16 + slot * (kDqk * 2) + (k + 2) * 128 + i * 16) : make_uint4(0, 0, 0, 0);
+        }
+        store_row_bf16(chunks + k * kChunkBytes, row, cur, valid16);
       }
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl.full[k]);
+    } else {
+#pragma unroll
+      for (int kc = 0; kc < 5; ++kc) {
+        const int k = 2 * kc + par;
+        if (k >= kNumChunks) break;
+        store_row<CB>(chunks + k * kChunkBytes, row, f[kc], CB == 4 || k == 8);
+        if (lane == 0) QMLA_TRACE(48 + warp * 5 + kc, it);
+      }
+    }
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      mbar_arrive(&ctl.tile_full);
+      QMLA_TRACE(32 + warp, it);
     }
     if (!ok) break;
-    if (ti.last) ++seg;
     ++it;
     sc.next();
     if (sc.valid()) {
@@ -438,89 +490,199 @@ __device__ void dequant_role(const Params& p, Sched sc, uint32_t chunks, uint32_
 }
 
 // ------------------------------------------------------------ MMA warp
-// The whole warp walks the schedule and waits; lane 0 issues the MMAs and the
-// commits (a commit tracks the MMAs issued by the committing thread).
+// Copies the query image of `unit` into shared memory with the bulk-copy
+// engine, completing on q_full through its transaction count.
 template <int HG>
-__device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint32_t qbase, Ctrl& ctl,
+__device__ __forceinline__ void issue_query(const Params& p, int unit, uint8_t* qsmem, Ctrl& ctl) {
+  constexpr uint32_t kBytes = Cfg<HG>::kQBytes;
+  mbar_arrive_expect_tx(&ctl.q_full, kBytes);
+  const uint8_t* src = p.qimg + static_cast<size_t>(unit) * kBytes;
+#pragma unroll 1
+  for (int k = 0; k < kNumChunks; ++k) bulk_g2s(qsmem + k * HG * 128, src + k * HG * 128, HG * 128, &ctl.q_full);
+}
+
+// One thread walks the schedule, waits, and issues the MMAs, the commits (a
+// commit tracks the MMAs issued by the committing thread) and the query
+// copies; the other lanes of the warp wait for it at the end. Descriptors
+// are advanced by adding (byte offset >> 4) to their start-address field.
+template <int HG>
+__device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint8_t* qsmem, Ctrl& ctl,
                          uint32_t tmem, int lane) {
-  constexpr uint32_t kIdQK = idesc_f16_f32(128, HG, false, false);
-  constexpr uint32_t kIdPV = idesc_f16_f32(128, HG, true, true);
-  constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
-  constexpr uint32_t kSboP = 8 * kRB;
-  const uint32_t ptile = chunks + 8 * kChunkBytes;
-  const uint32_t t_s = tmem + 4 * HG;
-  const bool leader = lane == 0;
-  uint32_t it = 0, seg = 0;
-  bool ok = true;
-  for (; ok && sc.valid(); sc.next()) {
-    const TileInfo ti = tile_info(sc, p);
-    if (ti.first && !(ok = wwait(&ctl.q_full, seg & 1u, ctl, kSiteMmaQFull, p.dev_err))) break;
-    // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576).
-    for (int k = 0; k < kNumChunks; ++k) {
-      if (!(ok = wwait(&ctl.full[k], it & 1u, ctl, kSiteMmaFull, p.dev_err))) break;
+  if (lane == 0) {
+    constexpr uint32_t kIdQK = idesc_f16_f32(128, HG, false, false);
+    constexpr uint32_t kIdPV = idesc_f16_f32(128, HG, true, true);
+    constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
+    constexpr uint32_t kSboP = 8 * kRB;
+    const uint32_t qbase = smem_u32(qsmem);
+    const uint32_t ptile = chunks + 8 * kChunkBytes;
+    const uint32_t t_s = tmem + 4 * HG;
+    const uint64_t qk_a0 = smem_desc(chunks, 16, 1024, SWZ_128B);
+    const uint64_t qk_b0 = smem_desc(qbase, 16, 1024, SWZ_128B);
+    const uint64_t pv_a0 = smem_desc(chunks, kChunkBytes, 1024, SWZ_128B);
+    const uint64_t pv_b0 = smem_desc(ptile, 16 * kSboP, kSboP, swz_mode_for_row(kRB));
+    uint32_t it = 0, seg = 0;
+    bool ok = true;
+    if (sc.valid()) issue_query<HG>(p, sc.u, qsmem, ctl);
+    for (; ok && sc.valid(); sc.next()) {
+      const TileInfo ti = tile_info(sc, p);
+      QMLA_TRACE(10, it);
+      if (ti.first && !(ok = wait_ok(mbar_wait(&ctl.q_full, seg & 1u, kWaitNs, &ctl.abort), kSiteMmaQFull, ctl, p.dev_err)))
+        break;
+      // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576).
+      if (!(ok = wait_ok(mbar_wait(&ctl.tile_full, it & 1u, kWaitNs, &ctl.abort), kSiteMmaFull, ctl, p.dev_err))) break;
       tc_fence_after();
-      if (leader) {
+      QMLA_TRACE(11, it);
+#pragma unroll 1
+      for (int k = 0; k < kNumChunks; ++k) {
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk) {
-          const uint64_t ad = smem_desc(chunks + k * kChunkBytes + kk * 32, 16, 1024, SWZ_128B);
-          const uint64_t bd = smem_desc(qbase + k * HG * 128 + kk * 32, 16, 1024, SWZ_128B);
+          const uint64_t ad = qk_a0 + static_cast<uint64_t>((k * kChunkBytes + kk * 32) >> 4);
+          const uint64_t bd = qk_b0 + static_cast<uint64_t>((k * HG * 128 + kk * 32) >> 4);
           umma_f16_ss(t_s, ad, bd, kIdQK, (k | kk) != 0 ? 1u : 0u);
         }
       }
-      __syncwarp();
-    }
-    if (!ok) break;
-    if (leader) {
       umma_commit(&ctl.s_full);
-      if (ti.last) umma_commit(&ctl.q_empty);
-    }
-    __syncwarp();
-    if (!(ok = wwait(&ctl.p_full, it & 1u, ctl, kSiteMmaPFull, p.dev_err))) break;
-    if (ti.first && seg > 0 && !(ok = wwait(&ctl.o_free, (seg - 1) & 1u, ctl, kSiteMmaOFree, p.dev_err))) break;
-    tc_fence_after();
-    // O^T[c, h] += sum_t C_hat[t, c] P^T[t, h], 4 x 128 channels, K = 128 tokens.
-    if (leader) {
+      QMLA_TRACE(12, it);
+      if (!(ok = wait_ok(mbar_wait(&ctl.p_full, it & 1u, kWaitNs, &ctl.abort), kSiteMmaPFull, ctl, p.dev_err))) break;
+      QMLA_TRACE(14, it);
+      if (ti.last) {
+        // The softmax only signals P after this tile's QK has completed, so the
+        // query tile is free: start copying the next segment's query now.
+        Sched nx = sc;
+        nx.next();
+        if (nx.valid()) issue_query<HG>(p, nx.u, qsmem, ctl);
+      }
+      if (ti.first && seg > 0 &&
+          !(ok = wait_ok(mbar_wait(&ctl.o_free, (seg - 1) & 1u, kWaitNs, &ctl.abort), kSiteMmaOFree, ctl, p.dev_err)))
+        break;
+      tc_fence_after();
+      // O^T[c, h] += sum_t C_hat[t, c] P^T[t, h], 4 x 128 channels, K = 128 tokens.
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t ad = smem_desc(chunks + 2 * i * kChunkBytes + kk * 2048, kChunkBytes, 1024, SWZ_128B);
-          const uint64_t bd = smem_desc(ptile + kk * 2 * kSboP, 16 * kSboP, kSboP, swz_mode_for_row(kRB));
+          const uint64_t ad = pv_a0 + static_cast<uint64_t>((2 * i * kChunkBytes + kk * 2048) >> 4);
+          const uint64_t bd = pv_b0 + static_cast<uint64_t>((kk * 2 * kSboP) >> 4);
           umma_f16_ss(tmem + i * HG, ad, bd, kIdPV, (ti.first && kk == 0) ? 0u : 1u);
         }
-        umma_commit(&ctl.empty[2 * i]);
-        umma_commit(&ctl.empty[2 * i + 1]);
       }
-      umma_commit(&ctl.empty[8]);
       umma_commit(&ctl.pv_done);
+      QMLA_TRACE(15, it);
+      ++it;
+      if (ti.last) ++seg;
     }
-    __syncwarp();
-    ++it;
-    if (ti.last) ++seg;
+    if (!ok) set_abort(ctl, p.dev_err);
+    // Every MMA and copy must have landed before TMEM and shared memory are released.
+    umma_commit(&ctl.fin);
+    wait_ok(mbar_wait(&ctl.fin, 0, kWaitNs, nullptr), kSiteMmaFin, ctl, p.dev_err);
   }
-  if (!ok) set_abort(ctl, p.dev_err);
-  // Every MMA must have landed before TMEM is released, aborted or not.
-  if (leader) umma_commit(&ctl.fin);
-  __syncwarp();
-  wait_ok(mbar_wait(&ctl.fin, 0, kWaitNs, nullptr), kSiteMmaFin, ctl, p.dev_err);
   __syncwarp();
 }
 
+// Column sums of a warp: v[j] summed over the 32 lanes for j = 0..15 by
+// recursive halving (16 shuffles); lane l ends with the total of element l >> 1.
+__device__ __forceinline__ float warp_colsum16(float (&v)[16], int lane) {
+  const bool b4 = lane & 16, b3 = lane & 8, b2 = lane & 4, b1 = lane & 2;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float send = b4 ? v[i] : v[i + 8];
+    const float keep = b4 ? v[i + 8] : v[i];
+    v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float send = b3 ? v[i] : v[i + 4];
+    const float keep = b3 ? v[i + 4] : v[i];
+    v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+  }
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const float send = b2 ? v[i] : v[i + 2];
+    const float keep = b2 ? v[i + 2] : v[i];
+    v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+  }
+  {
+    const float send = b1 ? v[0] : v[1];
+    const float keep = b1 ? v[1] : v[0];
+    v[0] = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+  }
+  return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 1);
+}
+
 // --------------------------------------------------------- softmax warps
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Tile max of the scaled scores per head into red[q4][h] (one warp's 32 rows).
+template <int HG>
+__device__ __forceinline__ void warp_tile_max(uint32_t t_s, float sl2, bool valid, Ctrl& ctl, int q4, int lane) {
+#pragma unroll
+  for (int c = 0; c < HG / 16; ++c) {
+    uint32_t r[16];
+    tmem_ld16(t_s + c * 16, r);
+    tmem_ld_wait();
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj) {
+      const float x = valid ? __uint_as_float(r[jj]) * sl2 : -INFINITY;
+      const float mx = warp_max_f32(x);
+      if (lane == jj) ctl.red[q4][c * 16 + jj] = mx;
+    }
+  }
+}
+
+// P^T[t, h] = 2^(S * scale * log2e - m_ref[h]) as fp16 into the P tile (row t)
+// and into pk; returns whether any of this thread's weights exceeds 2^8.
+template <int HG>
+__device__ __forceinline__ bool compute_p(uint32_t t_s, const float* m_ref, float sl2, bool valid, uint32_t ptile,
+                                          int row, uint32_t (&pk)[HG / 16][8]) {
+  constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
+  bool over = false;
+#pragma unroll
+  for (int c = 0; c < HG / 16; ++c) {
+    uint32_t r[16];
+    tmem_ld16(t_s + c * 16, r);
+    float m[16];
+#pragma unroll
+    for (int v4 = 0; v4 < 4; ++v4) {
+      const float4 mv = reinterpret_cast<const float4*>(m_ref)[c * 4 + v4];
+      m[4 * v4] = mv.x;
+      m[4 * v4 + 1] = mv.y;
+      m[4 * v4 + 2] = mv.z;
+      m[4 * v4 + 3] = mv.w;
+    }
+    tmem_ld_wait();
+#pragma unroll
+    for (int jj = 0; jj < 16; jj += 2) {
+      const float x0 = __uint_as_float(r[jj]) * sl2 - m[jj];
+      const float x1 = __uint_as_float(r[jj + 1]) * sl2 - m[jj + 1];
+      over |= valid && (fmaxf(x0, x1) > kRescaleLog2);
+      pk[c][jj >> 1] = valid ? pack_h2(ex2_approx(x0), ex2_approx(x1)) : 0u;
+    }
+    sts_v4(ptile + swz_off(row, 2 * c, kRB), pk[c][0], pk[c][1], pk[c][2], pk[c][3]);
+    sts_v4(ptile + swz_off(row, 2 * c + 1, kRB), pk[c][4], pk[c][5], pk[c][6], pk[c][7]);
+  }
+  return over;
+}
+
+// Softmax warps (TMEM lane quarter q4 = token rows 32 q4 .. 32 q4 + 31). Per
+// tile: P against the per-head reference max; only when a weight would exceed
+// 2^8 is the reference raised (O and the row sums rescaled, P recomputed).
+// The row sums of P live in TMEM columns [5 HG, 6 HG), one per head and row.
 template <int CB, int HG>
 __device__ void softmax_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ctl, uint32_t tmem,
                              int warp, int lane) {
+  constexpr int NC = HG / 16;
   const int q4 = warp & 3;
   const int row = q4 * 32 + lane;
   const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
   const uint32_t t_s = tmem + 4 * HG + lane_off;
   const uint32_t t_o = tmem + lane_off;
+  const uint32_t t_l = tmem + 5 * HG + lane_off;
   const uint32_t ptile = chunks + 8 * kChunkBytes;
-  constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
   const float sl2 = p.scale_log2;
-  float lsum[HG];
-#pragma unroll
-  for (int h = 0; h < HG; ++h) lsum[h] = 0.0f;
   uint32_t it = 0, gph[3] = {0, 0, 0};
   int seg_j0 = 0;
   bool ok = true;
@@ -530,110 +692,91 @@ __device__ void softmax_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& c
     const bool valid = row < ti.ntok;
     if (!(ok = wwait(&ctl.s_full, it & 1u, ctl, kSiteSmSFull, p.dev_err))) break;
     tc_fence_after();
-    // Pass 1: does any score exceed the reference max by more than 2^8?
-    bool need = ti.first;
-    if (!ti.first) {
-#pragma unroll
-      for (int c = 0; c < HG / 16; ++c) {
-        uint32_t r[16];
-        tmem_ld16(t_s + c * 16, r);
-        tmem_ld_wait();
-#pragma unroll
-        for (int jj = 0; jj < 16; ++jj)
-          need |= valid && (__uint_as_float(r[jj]) * sl2 > ctl.m_ref[c * 16 + jj] + kRescaleLog2);
-      }
+    if (lane == 0 && q4 == 0) QMLA_TRACE(16, it);
+    if (ti.first) {
+      // New segment: the reference is this tile's max.
+      warp_tile_max<HG>(t_s, sl2, valid, ctl, q4, lane);
+      if (!(ok = group_sync(&ctl.grp[1], gph[1], ctl, kSiteSmMax, p.dev_err))) break;
+      if (row < HG)
+        ctl.m_ref[row] = fmaxf(fmaxf(ctl.red[0][row], ctl.red[1][row]), fmaxf(ctl.red[2][row], ctl.red[3][row]));
+      if (!(ok = group_sync(&ctl.grp[2], gph[2], ctl, kSiteSmFinal, p.dev_err))) break;
     }
-    const uint32_t any = __any_sync(0xffffffffu, need);
+    uint32_t pk[NC][8];
+    const bool over = compute_p<HG>(t_s, ctl.m_ref, sl2, valid, ptile, row, pk);
     uint32_t* vote = ctl.vote[it & 1u];
+    const uint32_t any = __any_sync(0xffffffffu, over);
     if (lane == 0) vote[q4] = any;
     if (!(ok = group_sync(&ctl.grp[0], gph[0], ctl, kSiteSmVote, p.dev_err))) break;
+    if (lane == 0 && q4 == 0) QMLA_TRACE(17, it);
     if ((vote[0] | vote[1] | vote[2] | vote[3]) != 0u) {
-      // Tile max per head over the 128 tokens.
-#pragma unroll
-      for (int c = 0; c < HG / 16; ++c) {
-        uint32_t r[16];
-        tmem_ld16(t_s + c * 16, r);
-        tmem_ld_wait();
-#pragma unroll
-        for (int jj = 0; jj < 16; ++jj) {
-          const float x = valid ? __uint_as_float(r[jj]) * sl2 : -INFINITY;
-          const float mx = warp_max_f32(x);
-          if (lane == jj) ctl.red[q4][c * 16 + jj] = mx;
-        }
-      }
+      // Raise the reference to the running max; O and the row sums were
+      // accumulated against the old one and are scaled by alpha = 2^(m_old - m_new).
+      warp_tile_max<HG>(t_s, sl2, valid, ctl, q4, lane);
       if (!(ok = group_sync(&ctl.grp[1], gph[1], ctl, kSiteSmMax, p.dev_err))) break;
       if (row < HG) {
         const float mt = fmaxf(fmaxf(ctl.red[0][row], ctl.red[1][row]), fmaxf(ctl.red[2][row], ctl.red[3][row]));
         const float mo = ctl.m_ref[row];
-        const float mn = ti.first ? mt : fmaxf(mo, mt);
-        ctl.alpha[row] = ti.first ? 0.0f : exp2f(mo - mn);
+        const float mn = fmaxf(mo, mt);
+        ctl.alpha[row] = exp2f(mo - mn);
         ctl.m_ref[row] = mn;
       }
       if (!(ok = group_sync(&ctl.grp[2], gph[2], ctl, kSiteSmFinal, p.dev_err))) break;
-      if (ti.first) {
+      if (!(ok = wwait(&ctl.pv_done, (it - 1) & 1u, ctl, kSiteSmPvRescale, p.dev_err))) break;
+      tc_fence_after();
 #pragma unroll
-        for (int h = 0; h < HG; ++h) lsum[h] = 0.0f;
-      } else {
-        // O was accumulated against the old reference: wait for the previous
-        // PV to land, then scale every head's column by alpha.
-        if (!(ok = wwait(&ctl.pv_done, (it - 1) & 1u, ctl, kSiteSmPvRescale, p.dev_err))) break;
-        tc_fence_after();
+      for (int i = 0; i < 5; ++i) {  // O^T chunks 0..3 and the row sums (column block 5)
+        const uint32_t col = i < 4 ? i * HG : 5 * HG;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
+        for (int c = 0; c < NC; ++c) {
+          uint32_t r[16];
+          tmem_ld16(t_o + col + c * 16, r);
+          tmem_ld_wait();
 #pragma unroll
-          for (int c = 0; c < HG / 16; ++c) {
-            uint32_t r[16];
-            tmem_ld16(t_o + i * HG + c * 16, r);
-            tmem_ld_wait();
-#pragma unroll
-            for (int jj = 0; jj < 16; ++jj)
-              r[jj] = __float_as_uint(__uint_as_float(r[jj]) * ctl.alpha[c * 16 + jj]);
-            tmem_st16(t_o + i * HG + c * 16, r);
-          }
+          for (int jj = 0; jj < 16; ++jj) r[jj] = __float_as_uint(__uint_as_float(r[jj]) * ctl.alpha[c * 16 + jj]);
+          tmem_st16(t_o + col + c * 16, r);
         }
-        tmem_st_wait();
-#pragma unroll
-        for (int h = 0; h < HG; ++h) lsum[h] *= ctl.alpha[h];
       }
+      tmem_st_wait();
+      compute_p<HG>(t_s, ctl.m_ref, sl2, valid, ptile, row, pk);
+      if (lane == 0 && q4 == 0) QMLA_TRACE(18, it);
     }
-    // Pass 2: P^T[t, h] = 2^(S * scale * log2e - m_ref[h]) as fp16.
+    // Row sums of the fp16 weights the PV MMA multiplies with.
 #pragma unroll
-    for (int c = 0; c < HG / 16; ++c) {
+    for (int c = 0; c < NC; ++c) {
       uint32_t r[16];
-      tmem_ld16(t_s + c * 16, r);
-      tmem_ld_wait();
-      uint32_t pk[8];
+      if (!ti.first) {
+        tmem_ld16(t_l + c * 16, r);
+        tmem_ld_wait();
+      }
 #pragma unroll
       for (int jj = 0; jj < 16; jj += 2) {
-        const float p0 = valid ? exp2f(__uint_as_float(r[jj]) * sl2 - ctl.m_ref[c * 16 + jj]) : 0.0f;
-        const float p1 = valid ? exp2f(__uint_as_float(r[jj + 1]) * sl2 - ctl.m_ref[c * 16 + jj + 1]) : 0.0f;
-        const __half2 hp = __floats2half2_rn(p0, p1);
-        const float2 back = __half22float2(hp);
-        lsum[c * 16 + jj] += back.x;
-        lsum[c * 16 + jj + 1] += back.y;
-        pk[jj >> 1] = *reinterpret_cast<const uint32_t*>(&hp);
+        const float2 pf = __half22float2(*reinterpret_cast<const __half2*>(&pk[c][jj >> 1]));
+        r[jj] = __float_as_uint(ti.first ? pf.x : __uint_as_float(r[jj]) + pf.x);
+        r[jj + 1] = __float_as_uint(ti.first ? pf.y : __uint_as_float(r[jj + 1]) + pf.y);
       }
-      if constexpr (HG == 16) {
-        sts_v4(ptile + swz_off(row, 0, kRB), pk[0], pk[1], pk[2], pk[3]);
-        sts_v4(ptile + swz_off(row, 1, kRB), pk[4], pk[5], pk[6], pk[7]);
-      } else {
-        sts_v4(ptile + swz_off(row, 2 * c, kRB), pk[0], pk[1], pk[2], pk[3]);
-        sts_v4(ptile + swz_off(row, 2 * c + 1, kRB), pk[4], pk[5], pk[6], pk[7]);
-      }
+      tmem_st16(t_l + c * 16, r);
     }
+    tmem_st_wait();
     fence_proxy_async_smem();
     tc_fence_before();
     __syncwarp();
-    if (lane == 0) mbar_arrive(&ctl.p_full);
+    if (lane == 0) {
+      mbar_arrive(&ctl.p_full);
+      if (q4 == 0) QMLA_TRACE(19, it);
+    }
 
     if (ti.last) {
-      // Segment end: l[h] = sum over the 128 token rows; then read O^T.
+      // Segment end: l[h] = sum of the row sums over the 128 rows; then O^T.
 #pragma unroll
-      for (int h = 0; h < HG; ++h) {
-        float v = lsum[h];
+      for (int c = 0; c < NC; ++c) {
+        uint32_t r[16];
+        tmem_ld16(t_l + c * 16, r);
+        tmem_ld_wait();
+        float v[16];
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-        if (lane == 0) ctl.red[q4][h] = v;
+        for (int jj = 0; jj < 16; ++jj) v[jj] = __uint_as_float(r[jj]);
+        const float tot = warp_colsum16(v, lane);
+        if ((lane & 1) == 0) ctl.red[q4][c * 16 + (lane >> 1)] = tot;
       }
       if (!(ok = group_sync(&ctl.grp[1], gph[1], ctl, kSiteSmLsum, p.dev_err))) break;
       if (row < HG) ctl.alpha[row] = (ctl.red[0][row] + ctl.red[1][row]) + (ctl.red[2][row] + ctl.red[3][row]);
@@ -648,7 +791,7 @@ __device__ void softmax_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& c
         const int P = i * 128 + row;  // position in the reconstructed row
         const int ch = (P & ~7) + Perm<CB>::at(P & 7);
 #pragma unroll
-        for (int c = 0; c < HG / 16; ++c) {
+        for (int c = 0; c < NC; ++c) {
           uint32_t r[16];
           tmem_ld16(t_o + i * HG + c * 16, r);
           tmem_ld_wait();
@@ -677,7 +820,10 @@ __device__ void softmax_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& c
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl.o_free);
+      if (lane == 0) {
+        mbar_arrive(&ctl.o_free);
+        if (q4 == 0) QMLA_TRACE(20, it);
+      }
     }
     ++it;
   }
@@ -689,22 +835,19 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t chunks = smem_u32(smem);
-  const uint32_t qbase = chunks + kNumChunks * kChunkBytes;
+  uint8_t* qsmem = smem + kNumChunks * kChunkBytes;
   Ctrl& ctl = *reinterpret_cast<Ctrl*>(smem + kNumChunks * kChunkBytes + Cfg<HG>::kQBytes);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) QMLA_TRACE(22, 0);
 
   if (threadIdx.x == 0) {
-    for (int k = 0; k < kNumChunks; ++k) {
-      mbar_init(&ctl.full[k], 4);
-      mbar_init(&ctl.empty[k], 1);
-    }
+    mbar_init(&ctl.tile_full, kNumDqWarps);
     mbar_init(&ctl.s_full, 1);
     mbar_init(&ctl.p_full, 4);
     mbar_init(&ctl.pv_done, 1);
     mbar_init(&ctl.o_free, 4);
-    mbar_init(&ctl.q_empty, 1);
-    mbar_init(&ctl.q_full, kNumDqWarps);
+    mbar_init(&ctl.q_full, 1);
     mbar_init(&ctl.fin, 1);
     for (int i = 0; i < 3; ++i) mbar_init(&ctl.grp[i], 4);
     ctl.abort = 0u;
@@ -722,11 +865,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   Sched sc;
   sc.init(p.prefix, p.batch * p.n_hg, blockIdx.x, gridDim.x);
   if (warp < kNumDqWarps) {
-    dequant_role<CB, HG>(p, sc, chunks, qbase, ctl, warp, lane);
+    dequant_role<CB, HG>(p, sc, chunks, ctl, warp, lane);
   } else if (warp < kMmaWarp) {
     softmax_role<CB, HG>(p, sc, chunks, ctl, tmem, warp, lane);
   } else {
-    mma_role<HG>(p, sc, chunks, qbase, ctl, tmem, lane);
+    mma_role<HG>(p, sc, chunks, qsmem, ctl, tmem, lane);
   }
   tc_fence_before();
   __syncthreads();
@@ -734,30 +877,45 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
     tc_fence_after();
     tmem_dealloc(tmem, Cfg<HG>::kTmemCols);
   }
+  if (threadIdx.x == 0) QMLA_TRACE(23, 0);
 }
 
-// ------------------------------------------------------------ plan / combine
-__global__ void __launch_bounds__(1024) plan_kernel(const int32_t* __restrict__ seq_lens, int batch,
-                                                    int n_hg, int max_blocks, int32_t* __restrict__ prefix,
-                                                    uint32_t* dev_err) {
+// ------------------------------------------------------------ prep / combine
+constexpr int kPrepThreads = 1024;
+
+// Block 0: tile prefix over units (u = b * n_hg + hg), tiles = ceil(len / 128).
+// Blocks 1..: one query-image piece (16 bytes) per thread.
+template <int CB, int HG>
+__global__ void __launch_bounds__(kPrepThreads) prep_kernel(const Params p) {
+  if (blockIdx.x > 0) {
+    const long long idx = static_cast<long long>(blockIdx.x - 1) * kPrepThreads + threadIdx.x;
+    constexpr int kPieces = kNumChunks * HG * 8;
+    const long long units = static_cast<long long>(p.batch) * p.n_hg;
+    if (idx >= units * kPieces) return;
+    const int u = static_cast<int>(idx / kPieces);
+    const int b = u / p.n_hg;
+    query_piece<CB, HG>(p, p.qimg + static_cast<size_t>(u) * Cfg<HG>::kQBytes, b, (u - b * p.n_hg) * HG,
+                        static_cast<int>(idx - static_cast<long long>(u) * kPieces));
+    return;
+  }
   __shared__ int warp_sums[32];
   __shared__ int carry;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int nwarps = blockDim.x >> 5;
   if (threadIdx.x == 0) carry = 0;
   __syncthreads();
-  for (int base = 0; base < batch; base += blockDim.x) {
+  for (int base = 0; base < p.batch; base += blockDim.x) {
     const int b = base + threadIdx.x;
     int tiles = 0;
-    if (b < batch) {
-      int len = seq_lens[b];
-      if (len < 0 || len > max_blocks * kBlockTokens) {
-        report(dev_err, QMLA_DEVERR_BAD_POSITION);
+    if (b < p.batch) {
+      int len = p.seq_lens[b];
+      if (len < 0 || len > p.max_blocks * kBlockTokens) {
+        report(p.dev_err, QMLA_DEVERR_BAD_POSITION);
         len = 0;
       }
       tiles = (len + kTileTokens - 1) / kTileTokens;
     }
-    const int v = tiles * n_hg;
+    const int v = tiles * p.n_hg;
     int x = v;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
@@ -767,24 +925,24 @@ __global__ void __launch_bounds__(1024) plan_kernel(const int32_t* __restrict__ 
     if (lane == 31) warp_sums[warp] = x;
     __syncthreads();
     if (warp == 0) {
-      int s = lane < nwarps ? warp_sums[lane] : 0;
+      int sw = lane < nwarps ? warp_sums[lane] : 0;
 #pragma unroll
       for (int off = 1; off < 32; off <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, s, off);
-        if (lane >= off) s += y;
+        const int y = __shfl_up_sync(0xffffffffu, sw, off);
+        if (lane >= off) sw += y;
       }
-      warp_sums[lane] = s;
+      warp_sums[lane] = sw;
     }
     __syncthreads();
     const int excl = carry + (warp > 0 ? warp_sums[warp - 1] : 0) + x - v;
-    if (b < batch) {
-      for (int hg = 0; hg < n_hg; ++hg) prefix[b * n_hg + hg] = excl + hg * tiles;
+    if (b < p.batch) {
+      for (int hg = 0; hg < p.n_hg; ++hg) p.prefix_w[b * p.n_hg + hg] = excl + hg * tiles;
     }
     __syncthreads();
     if (threadIdx.x == blockDim.x - 1) carry = excl + v;
     __syncthreads();
   }
-  if (threadIdx.x == 0) prefix[batch * n_hg] = carry;
+  if (threadIdx.x == 0) p.prefix_w[p.batch * p.n_hg] = carry;
 }
 
 // First tile of CTA c's range, and the CTA whose range holds tile t.
@@ -795,53 +953,52 @@ __device__ __forceinline__ int cta_of(int t, int T, int grid) {
   return static_cast<int>((static_cast<long long>(t + 1) * grid - 1) / T);
 }
 
+// One block per (unit, head): merges that head's partials with the App. C.5
+// rule; each thread owns 4 of the 512 channels.
 template <int HG>
-__global__ void __launch_bounds__(256) combine_kernel(const Params p) {
+__global__ void __launch_bounds__(128) combine_kernel(const Params p) {
   const int u = blockIdx.x;
+  const int h = blockIdx.y;
   const int units = p.batch * p.n_hg;
   const int b = u / p.n_hg;
   const int h0 = (u - b * p.n_hg) * HG;
-  const int nh = min(HG, p.heads - h0);
+  if (h0 + h >= p.heads) return;
   const int P0 = p.prefix[u], P1 = p.prefix[u + 1], T = p.prefix[units];
-  float* out = p.out + (static_cast<size_t>(b) * p.heads + h0) * kDc;
+  float4* out = reinterpret_cast<float4*>(p.out + (static_cast<size_t>(b) * p.heads + h0 + h) * kDc);
+  const int q = threadIdx.x;
   if (P0 == P1) {
-    for (int idx = threadIdx.x; idx < nh * kDc; idx += blockDim.x) out[idx] = 0.0f;
-    if (p.lse != nullptr && threadIdx.x < nh) p.lse[static_cast<size_t>(b) * p.heads + h0 + threadIdx.x] = -INFINITY;
+    out[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (p.lse != nullptr && q == 0) p.lse[static_cast<size_t>(b) * p.heads + h0 + h] = -INFINITY;
     return;
   }
   const int c0 = cta_of(P0, T, p.grid), c1 = cta_of(P1 - 1, T, p.grid);
   if (c0 == c1) return;  // one CTA covered the whole unit and wrote the result
-  for (int idx = threadIdx.x; idx < nh * (kDc / 4); idx += blockDim.x) {
-    const int h = idx / (kDc / 4);
-    const int q = idx - h * (kDc / 4);
-    // CTAs between c0 and c1 with an empty range wrote no partial.
-    float M = -INFINITY;
-    for (int c = c0; c <= c1; ++c) {
-      if (cta_start(c, T, p.grid) == cta_start(c + 1, T, p.grid)) continue;
-      M = fmaxf(M, p.part_ml[((static_cast<size_t>(c) + u) * HG + h) * 2]);
-    }
-    float s = 0.0f;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int c = c0; c <= c1; ++c) {
-      if (cta_start(c, T, p.grid) == cta_start(c + 1, T, p.grid)) continue;
-      const size_t pi = (static_cast<size_t>(c) + u) * HG + h;
-      const float w = exp2f(p.part_ml[pi * 2] - M);
-      s += w * p.part_ml[pi * 2 + 1];
-      const float4 o = reinterpret_cast<const float4*>(p.part_o + pi * kDc)[q];
-      acc.x += w * o.x;
-      acc.y += w * o.y;
-      acc.z += w * o.z;
-      acc.w += w * o.w;
-    }
-    const float inv = 1.0f / s;
-    reinterpret_cast<float4*>(out + static_cast<size_t>(h) * kDc)[q] =
-        make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
-    if (q == 0 && p.lse != nullptr) p.lse[static_cast<size_t>(b) * p.heads + h0 + h] = (M + log2f(s)) * kLn2;
+  // CTAs between c0 and c1 with an empty range wrote no partial.
+  float M = -INFINITY;
+  for (int c = c0; c <= c1; ++c) {
+    if (cta_start(c, T, p.grid) == cta_start(c + 1, T, p.grid)) continue;
+    M = fmaxf(M, p.part_ml[((static_cast<size_t>(c) + u) * HG + h) * 2]);
   }
+  float s = 0.0f;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int c = c0; c <= c1; ++c) {
+    if (cta_start(c, T, p.grid) == cta_start(c + 1, T, p.grid)) continue;
+    const size_t pi = (static_cast<size_t>(c) + u) * HG + h;
+    const float w = exp2f(p.part_ml[pi * 2] - M);
+    s += w * p.part_ml[pi * 2 + 1];
+    const float4 o = reinterpret_cast<const float4*>(p.part_o + pi * kDc)[q];
+    acc.x += w * o.x;
+    acc.y += w * o.y;
+    acc.z += w * o.z;
+    acc.w += w * o.w;
+  }
+  const float inv = 1.0f / s;
+  out[q] = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+  if (q == 0 && p.lse != nullptr) p.lse[static_cast<size_t>(b) * p.heads + h0 + h] = (M + log2f(s)) * kLn2;
 }
 
 template <int CB, int HG>
-cudaError_t launch_impl(const Params& prm, cudaStream_t stream) {
+cudaError_t launch_impl(const Params& prm, cudaStream_t stream, cudaEvent_t ev0, cudaEvent_t ev1) {
   static int configured_device = -1;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -851,18 +1008,24 @@ cudaError_t launch_impl(const Params& prm, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     configured_device = dev;
   }
+  const long long units = static_cast<long long>(prm.batch) * prm.n_hg;
+  const long long pieces = units * kNumChunks * HG * 8;
+  const unsigned prep_blocks = static_cast<unsigned>(1 + (pieces + kPrepThreads - 1) / kPrepThreads);
+  prep_kernel<CB, HG><<<prep_blocks, kPrepThreads, 0, stream>>>(prm);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if (ev0 != nullptr && (e = cudaEventRecord(ev0, stream)) != cudaSuccess) return e;
   decode_main<CB, HG><<<prm.grid, kThreads, Cfg<HG>::kSmem, stream>>>(prm);
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  combine_kernel<HG><<<prm.batch * prm.n_hg, 256, 0, stream>>>(prm);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if (ev1 != nullptr && (e = cudaEventRecord(ev1, stream)) != cudaSuccess) return e;
+  combine_kernel<HG><<<dim3(static_cast<unsigned>(units), HG), 128, 0, stream>>>(prm);
   return cudaGetLastError();
 }
 
 template <int CB>
-cudaError_t launch_hg(int hg, const Params& prm, cudaStream_t stream) {
-  if (hg == 16) return launch_impl<CB, 16>(prm, stream);
-  if (hg == 32) return launch_impl<CB, 32>(prm, stream);
-  return launch_impl<CB, 64>(prm, stream);
+cudaError_t launch_hg(int hg, const Params& prm, cudaStream_t stream, cudaEvent_t ev0, cudaEvent_t ev1) {
+  if (hg == 16) return launch_impl<CB, 16>(prm, stream, ev0, ev1);
+  if (hg == 32) return launch_impl<CB, 32>(prm, stream, ev0, ev1);
+  return launch_impl<CB, 64>(prm, stream, ev0, ev1);
 }
 
 }  // namespace
@@ -878,7 +1041,8 @@ DecodeWorkspace decode_workspace_layout(int batch, int heads, int grid) {
   w.part_o_off = up((units + 1) * sizeof(int32_t));
   const size_t nparts = static_cast<size_t>(grid) + units;
   w.part_ml_off = w.part_o_off + up(nparts * hg * kDc * sizeof(float));
-  w.total = w.part_ml_off + up(nparts * hg * 2 * sizeof(float));
+  w.qimg_off = w.part_ml_off + up(nparts * hg * 2 * sizeof(float));
+  w.total = w.qimg_off + up(units * kNumChunks * hg * 128);
   return w;
 }
 
@@ -904,14 +1068,19 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
   prm.prefix_w = reinterpret_cast<int32_t*>(ws + w.prefix_off);
   prm.part_o = reinterpret_cast<float*>(ws + w.part_o_off);
   prm.part_ml = reinterpret_cast<float*>(ws + w.part_ml_off);
+  prm.qimg = ws + w.qimg_off;
   prm.dev_err = a.dev_err;
   prm.grid = a.grid;
-  plan_kernel<<<1, 1024, 0, stream>>>(a.seq_lens, a.batch, prm.n_hg, a.max_blocks, prm.prefix_w, a.dev_err);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  if (a.cache_kind == 4) return launch_hg<4>(hg, prm, stream);
-  if (a.cache_kind == 2) return launch_hg<2>(hg, prm, stream);
-  return launch_hg<16>(hg, prm, stream);
+  if (a.cache_kind == 4) return launch_hg<4>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
+  if (a.cache_kind == 2) return launch_hg<2>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
+  return launch_hg<16>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
 }
+
+#ifdef QMLA_TRACE_BUILD
+cudaError_t set_trace_buffer(void* buf) {
+  unsigned long long* p = static_cast<unsigned long long*>(buf);
+  return cudaMemcpyToSymbol(g_trace, &p, sizeof(p));
+}
+#endif
 
 }  // namespace qmla

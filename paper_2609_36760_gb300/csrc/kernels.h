@@ -21,7 +21,7 @@ int head_group_size(int heads);
 
 // Workspace carve-up of the decode path for `grid` CTAs.
 struct DecodeWorkspace {
-  size_t prefix_off, part_o_off, part_ml_off, total;
+  size_t prefix_off, part_o_off, part_ml_off, qimg_off, total;
 };
 DecodeWorkspace decode_workspace_layout(int batch, int heads, int grid);
 
@@ -41,7 +41,14 @@ struct DecodeArgs {
   void* workspace;
   uint32_t* dev_err;
   int grid;  // CTAs of the main kernel (one per SM)
+  cudaEvent_t ev_before_main = nullptr;  // optional, recorded around the main kernel
+  cudaEvent_t ev_after_main = nullptr;
 };
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
+
+#ifdef QMLA_TRACE_BUILD
+// Trace builds only: device buffer of [8 CTAs][96 events][32 tiles] u64 clock64 stamps.
+cudaError_t set_trace_buffer(void* buf);
+#endif
 
 }  // namespace qmla

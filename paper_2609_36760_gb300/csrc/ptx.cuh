@@ -40,13 +40,26 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t by
       "r"(bytes)
       : "memory");
 }
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+// Non-blocking probe of a phase.
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
-      "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
       : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Potentially blocking probe: the thread sleeps until the phase completes or
+// about 100 us pass, so waiting warps do not take issue slots from working ones.
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(100000u)
       : "memory");
   return ok != 0;
 }
@@ -55,14 +68,12 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // non-zero first.
 __device__ __forceinline__ int mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns,
                                          const volatile uint32_t* abort) {
-  if (mbar_try_wait(bar, parity)) return 1;
+  if (mbar_test(bar, parity)) return 1;
   const uint64_t t0 = globaltimer_ns();
-  for (uint32_t it = 1;; ++it) {
+  for (;;) {
     if (mbar_try_wait(bar, parity)) return 1;
-    if ((it & 63u) == 0u) {
-      if (abort != nullptr && *abort != 0u) return -1;
-      if (globaltimer_ns() - t0 > limit_ns) return 0;
-    }
+    if (abort != nullptr && *abort != 0u) return -1;
+    if (globaltimer_ns() - t0 > limit_ns) return 0;
   }
 }
 

@@ -106,10 +106,16 @@ def test_split_units_and_combine():
 def test_same_answer_at_any_split():
     # The same sequence decoded alone (few splits) and next to long neighbours
     # (many splits) agrees to fp32 accumulation-order noise.
-    w_alone = W.small_workload("a", batch=1, heads=64, lengths=(5000,), seed=51)
-    c1, out1, _ = run_case(w_alone)
     w_many = W.small_workload("a", batch=4, heads=64, lengths=(5000, 60000, 60000, 60000), seed=51)
-    c2, out2, _ = run_case(w_many)
+    w_alone = W.small_workload("a", batch=1, heads=64, lengths=(5000,), seed=51)
+    ql, qp = W.queries(w_many, 0)
+    c1 = Case(w_alone)
+    c1.prefill_all()
+    out1, _ = c1.decode(0, queries=(ql[:1].contiguous(), qp[:1].contiguous()))
+    c2 = Case(w_many)
+    c2.prefill_all()
+    out2, _ = c2.decode(0, queries=(ql, qp))
+    assert c1.dev_error() == 0 and c2.dev_error() == 0
     assert np.max(np.abs(out1[0] - out2[0])) <= 1e-4
 
 
