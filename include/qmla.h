@@ -165,6 +165,38 @@ int qmla_mla_decode_bf16cache(const void* pool_dev, int num_blocks, const uint16
  * cudaEventElapsedTime. Pass NULL, NULL to stop. Always returns QMLA_OK. */
 int qmla_set_profile_events(void* before_main, void* after_main);
 
+/* Bytes of the fixed device scratch array qmla_mla_decode_static uses
+ * (32 MiB). */
+size_t qmla_static_scratch_bytes(void);
+
+/*
+ * qmla_mla_decode without a workspace argument, for callers that cannot
+ * allocate device memory where they call it (for example code running inside
+ * an allocator-free region of a serving loop, or a host library that is
+ * handed finished buffers and must not call cudaMalloc, whose implicit
+ * synchronisation and memory growth it does not control). The paper has no
+ * counterpart; this is a deployment convenience.
+ *
+ * Inputs, outputs and results are exactly those of qmla_mla_decode. The
+ * scratch the decode needs lives in one file-scope device array of
+ * qmla_static_scratch_bytes() bytes that every GPU loading this library holds
+ * until the process exits. Nothing is allocated or freed by this call.
+ * - The first call on a device looks up that array's device address
+ *   (cudaGetSymbolAddress) with the device current; make that first call
+ *   before capturing any stream.
+ * - Returns QMLA_ERR_WORKSPACE_TOO_SMALL when batch x heads need more scratch
+ *   than the array holds (qmla_decode_workspace_bytes(batch, heads) >
+ *   qmla_static_scratch_bytes(); e.g. up to 32 sequences at 128 heads).
+ * - Every call shares the array, which keeps the last call's contents;
+ *   nothing in it needs to start at zero (each call rewrites everything it
+ *   reads). Calls whose work overlaps on the GPU (different streams, or
+ *   different host threads on one device) race on it: serialise them.
+ */
+int qmla_mla_decode_static(const void* pool_dev, int c_bits, int num_blocks, const uint16_t* q_latent_dev,
+                           const uint16_t* q_pe_dev, int batch, int heads, const int32_t* block_table_dev,
+                           int max_blocks, const int32_t* seq_lens_dev, float softmax_scale, float* out_dev,
+                           float* lse_dev, uint32_t* dev_err_dev, qmla_stream_t stream);
+
 /* Copies the device error word to *host_out after synchronising `stream`. */
 int qmla_read_dev_err(const uint32_t* dev_err_dev, uint32_t* host_out, qmla_stream_t stream);
 

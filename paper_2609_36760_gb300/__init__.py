@@ -64,6 +64,9 @@ def lib():
     L.qmla_status_string.argtypes, L.qmla_status_string.restype = [i32], ctypes.c_char_p
     L.qmla_num_sms.argtypes, L.qmla_num_sms.restype = [], i32
     L.qmla_set_profile_events.argtypes, L.qmla_set_profile_events.restype = [vp, vp], i32
+    L.qmla_static_scratch_bytes.argtypes, L.qmla_static_scratch_bytes.restype = [], sz
+    L.qmla_mla_decode_static.argtypes = [vp, i32, i32, vp, vp, i32, i32, vp, i32, vp, f32, vp, vp, vp, vp]
+    L.qmla_mla_decode_static.restype = i32
     _lib = L
     return L
 
@@ -146,6 +149,22 @@ def mla_decode_bf16cache(pool: torch.Tensor, q_latent: torch.Tensor, q_pe: torch
                                          workspace.numel() * workspace.element_size(), _ptr(dev_err),
                                          _stream(stream))
     _check("qmla_mla_decode_bf16cache", st)
+
+
+def mla_decode_static(pool: torch.Tensor, c_bits: int, q_latent: torch.Tensor, q_pe: torch.Tensor,
+                      block_table: torch.Tensor, seq_lens: torch.Tensor, softmax_scale: float, out: torch.Tensor,
+                      lse: torch.Tensor | None, dev_err: torch.Tensor, stream=None) -> None:
+    """qmla_mla_decode_static: qmla_mla_decode for callers that cannot allocate a
+    workspace; uses the library's fixed device scratch (see include/qmla.h)."""
+    B, H = q_latent.shape[0], q_latent.shape[1]
+    st = lib().qmla_mla_decode_static(_ptr(pool), c_bits, pool.shape[0], _ptr(q_latent), _ptr(q_pe), B, H,
+                                      _ptr(block_table), block_table.shape[1], _ptr(seq_lens),
+                                      float(softmax_scale), _ptr(out), _ptr(lse), _ptr(dev_err), _stream(stream))
+    _check("qmla_mla_decode_static", st)
+
+
+def static_scratch_bytes() -> int:
+    return int(lib().qmla_static_scratch_bytes())
 
 
 def set_profile_events(before_main: torch.cuda.Event | None, after_main: torch.cuda.Event | None) -> None:

@@ -103,6 +103,10 @@ int decode_common(const void* pool, int kind, int num_blocks, const uint16_t* q_
 
 }  // namespace
 
+namespace qmla {
+void record_cuda_error(int err) { g_last_cuda_error = err; }
+}  // namespace qmla
+
 extern "C" {
 
 size_t qmla_block_bytes(int c_bits) {

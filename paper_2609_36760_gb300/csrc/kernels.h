@@ -46,6 +46,9 @@ struct DecodeArgs {
 };
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
 
+// Records a failed CUDA call for qmla_last_cuda_error (calling thread).
+void record_cuda_error(int err);
+
 #ifdef QMLA_TRACE_BUILD
 // Trace builds only: device buffer of [8 CTAs][96 events][32 tiles] u64 clock64 stamps.
 cudaError_t set_trace_buffer(void* buf);
