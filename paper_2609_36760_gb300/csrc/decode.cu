@@ -58,11 +58,12 @@ constexpr float kLn2 = 0.6931471805599453f;
 // for trace builds (-DQMLA_TRACE_BUILD); see qmla_trace_set in api.cu.
 #ifdef QMLA_TRACE_BUILD
 constexpr int kTraceCtas = 8, kTraceEvents = 96, kTraceTiles = 32;
-__device__ unsigned long long* g_trace = nullptr;
+// The buffer pointer travels in the kernel parameters (constant bank), so an
+// event costs one clock read and one global store, no load.
 #define QMLA_TRACE(ev, tile)                                                                     \
   do {                                                                                           \
-    if (g_trace != nullptr && blockIdx.x < kTraceCtas && (tile) < kTraceTiles)                   \
-      g_trace[(static_cast<size_t>(blockIdx.x) * kTraceEvents + (ev)) * kTraceTiles + (tile)] = \
+    if (p.trace != nullptr && blockIdx.x < kTraceCtas && (tile) < kTraceTiles)                   \
+      p.trace[(static_cast<size_t>(blockIdx.x) * kTraceEvents + (ev)) * kTraceTiles + (tile)] = \
           clock64();                                                                             \
   } while (0)
 #else
@@ -90,6 +91,7 @@ struct Params {
   uint8_t* qimg;   // [units][9][HG][128 B]: swizzled fp16 query tiles
   uint32_t* dev_err;
   int grid;
+  unsigned long long* trace;  // trace builds only: per-CTA event clocks, else null
 };
 
 struct __align__(16) Ctrl {
@@ -194,20 +196,17 @@ __device__ __forceinline__ bool wait_ok(int r, uint32_t site, Ctrl& c, uint32_t*
   }
   return r == 1;
 }
-// Warp-uniform bounded wait: lane 0 polls (mbarrier polls share the
-// shared-memory pipe with the tensor core's operand reads, so one poller per
-// warp keeps them cheap), then every lane acquires the completed phase once.
+// Warp-uniform bounded wait: every lane waits on the barrier itself. Letting
+// one lane poll while the others sit at a warp-synchronising instruction was
+// measured to be much slower on sm_103a: the parked warp delayed the draining
+// of other warps' shared-memory stores by thousands of cycles, and its own
+// wake-up after the phase completed took ~2k cycles.
 __device__ __forceinline__ bool wwait(uint64_t* bar, uint32_t parity, Ctrl& c, uint32_t site,
                                       uint32_t* dev_err) {
-  int r = 1;
-  if ((threadIdx.x & 31) == 0) r = mbar_wait(bar, parity, kWaitNs, &c.abort);
-  r = __shfl_sync(0xffffffffu, r, 0);
-  if (r == 1) {
-    (void)mbar_test(bar, parity);
-  } else if ((threadIdx.x & 31) == 0) {
-    wait_ok(r, site, c, dev_err);
-  }
-  return r == 1;
+  const int r = mbar_wait(bar, parity, kWaitNs, &c.abort);
+  const bool all_ok = __all_sync(0xffffffffu, r == 1);
+  if (r == 0) wait_ok(r, site, c, dev_err);
+  return all_ok;
 }
 // Barrier among the four softmax warps (one arrive per warp), bounded.
 __device__ __forceinline__ bool group_sync(uint64_t* bar, uint32_t& phase, Ctrl& c, uint32_t site,
@@ -501,36 +500,36 @@ __device__ __forceinline__ void issue_query(const Params& p, int unit, uint8_t* 
   for (int k = 0; k < kNumChunks; ++k) bulk_g2s(qsmem + k * HG * 128, src + k * HG * 128, HG * 128, &ctl.q_full);
 }
 
-// One thread walks the schedule, waits, and issues the MMAs, the commits (a
-// commit tracks the MMAs issued by the committing thread) and the query
-// copies; the other lanes of the warp wait for it at the end. Descriptors
-// are advanced by adding (byte offset >> 4) to their start-address field.
+// The MMA warp walks the schedule and waits on every lane; one elected lane
+// issues the MMAs, the commits (a commit tracks the MMAs issued by the
+// committing thread) and the query copies. Descriptors are advanced by adding
+// (byte offset >> 4) to their start-address field.
 template <int HG>
 __device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint8_t* qsmem, Ctrl& ctl,
                          uint32_t tmem, int lane) {
-  if (lane == 0) {
-    constexpr uint32_t kIdQK = idesc_f16_f32(128, HG, false, false);
-    constexpr uint32_t kIdPV = idesc_f16_f32(128, HG, true, true);
-    constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
-    constexpr uint32_t kSboP = 8 * kRB;
-    const uint32_t qbase = smem_u32(qsmem);
-    const uint32_t ptile = chunks + 8 * kChunkBytes;
-    const uint32_t t_s = tmem + 4 * HG;
-    const uint64_t qk_a0 = smem_desc(chunks, 16, 1024, SWZ_128B);
-    const uint64_t qk_b0 = smem_desc(qbase, 16, 1024, SWZ_128B);
-    const uint64_t pv_a0 = smem_desc(chunks, kChunkBytes, 1024, SWZ_128B);
-    const uint64_t pv_b0 = smem_desc(ptile, 16 * kSboP, kSboP, swz_mode_for_row(kRB));
-    uint32_t it = 0, seg = 0;
-    bool ok = true;
-    if (sc.valid()) issue_query<HG>(p, sc.u, qsmem, ctl);
-    for (; ok && sc.valid(); sc.next()) {
-      const TileInfo ti = tile_info(sc, p);
-      QMLA_TRACE(10, it);
-      if (ti.first && !(ok = wait_ok(mbar_wait(&ctl.q_full, seg & 1u, kWaitNs, &ctl.abort), kSiteMmaQFull, ctl, p.dev_err)))
-        break;
-      // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576).
-      if (!(ok = wait_ok(mbar_wait(&ctl.tile_full, it & 1u, kWaitNs, &ctl.abort), kSiteMmaFull, ctl, p.dev_err))) break;
-      tc_fence_after();
+  const bool leader = lane == 0;
+  constexpr uint32_t kIdQK = idesc_f16_f32(128, HG, false, false);
+  constexpr uint32_t kIdPV = idesc_f16_f32(128, HG, true, true);
+  constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
+  constexpr uint32_t kSboP = 8 * kRB;
+  const uint32_t qbase = smem_u32(qsmem);
+  const uint32_t ptile = chunks + 8 * kChunkBytes;
+  const uint32_t t_s = tmem + 4 * HG;
+  const uint64_t qk_a0 = smem_desc(chunks, 16, 1024, SWZ_128B);
+  const uint64_t qk_b0 = smem_desc(qbase, 16, 1024, SWZ_128B);
+  const uint64_t pv_a0 = smem_desc(chunks, kChunkBytes, 1024, SWZ_128B);
+  const uint64_t pv_b0 = smem_desc(ptile, 16 * kSboP, kSboP, swz_mode_for_row(kRB));
+  uint32_t it = 0, seg = 0;
+  bool ok = true;
+  if (sc.valid() && leader) issue_query<HG>(p, sc.u, qsmem, ctl);
+  for (; ok && sc.valid(); sc.next()) {
+    const TileInfo ti = tile_info(sc, p);
+    if (leader) QMLA_TRACE(10, it);
+    if (ti.first && !(ok = wwait(&ctl.q_full, seg & 1u, ctl, kSiteMmaQFull, p.dev_err))) break;
+    // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576).
+    if (!(ok = wwait(&ctl.tile_full, it & 1u, ctl, kSiteMmaFull, p.dev_err))) break;
+    tc_fence_after();
+    if (leader) {
       QMLA_TRACE(11, it);
 #pragma unroll 1
       for (int k = 0; k < kNumChunks; ++k) {
@@ -543,19 +542,22 @@ __device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint8_t* qs
       }
       umma_commit(&ctl.s_full);
       QMLA_TRACE(12, it);
-      if (!(ok = wait_ok(mbar_wait(&ctl.p_full, it & 1u, kWaitNs, &ctl.abort), kSiteMmaPFull, ctl, p.dev_err))) break;
-      QMLA_TRACE(14, it);
-      if (ti.last) {
-        // The softmax only signals P after this tile's QK has completed, so the
-        // query tile is free: start copying the next segment's query now.
-        Sched nx = sc;
-        nx.next();
-        if (nx.valid()) issue_query<HG>(p, nx.u, qsmem, ctl);
-      }
-      if (ti.first && seg > 0 &&
-          !(ok = wait_ok(mbar_wait(&ctl.o_free, (seg - 1) & 1u, kWaitNs, &ctl.abort), kSiteMmaOFree, ctl, p.dev_err)))
-        break;
-      tc_fence_after();
+    }
+    __syncwarp();
+    if (!(ok = wwait(&ctl.p_full, it & 1u, ctl, kSiteMmaPFull, p.dev_err))) break;
+    if (leader) QMLA_TRACE(14, it);
+    if (ti.last && leader) {
+      // The softmax only signals P after this tile's QK has completed, so the
+      // query tile is free: start copying the next segment's query now.
+      Sched nx = sc;
+      nx.next();
+      if (nx.valid()) issue_query<HG>(p, nx.u, qsmem, ctl);
+    }
+    if (ti.first && seg > 0 &&
+        !(ok = wwait(&ctl.o_free, (seg - 1) & 1u, ctl, kSiteMmaOFree, p.dev_err)))
+      break;
+    tc_fence_after();
+    if (leader) {
       // O^T[c, h] += sum_t C_hat[t, c] P^T[t, h], 4 x 128 channels, K = 128 tokens.
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
@@ -568,14 +570,17 @@ __device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint8_t* qs
       }
       umma_commit(&ctl.pv_done);
       QMLA_TRACE(15, it);
-      ++it;
-      if (ti.last) ++seg;
     }
-    if (!ok) set_abort(ctl, p.dev_err);
-    // Every MMA and copy must have landed before TMEM and shared memory are released.
-    umma_commit(&ctl.fin);
-    wait_ok(mbar_wait(&ctl.fin, 0, kWaitNs, nullptr), kSiteMmaFin, ctl, p.dev_err);
+    __syncwarp();
+    ++it;
+    if (ti.last) ++seg;
   }
+  if (!ok && leader) set_abort(ctl, p.dev_err);
+  // Every MMA and copy must have landed before TMEM and shared memory are released.
+  // This wait ignores the abort flag: TMEM may only be released once they have.
+  if (leader) umma_commit(&ctl.fin);
+  __syncwarp();
+  wait_ok(mbar_wait(&ctl.fin, 0, kWaitNs, nullptr), kSiteMmaFin, ctl, p.dev_err);
   __syncwarp();
 }
 
@@ -1030,6 +1035,10 @@ cudaError_t launch_hg(int hg, const Params& prm, cudaStream_t stream, cudaEvent_
 
 }  // namespace
 
+#ifdef QMLA_TRACE_BUILD
+unsigned long long* g_trace_buf = nullptr;  // set by set_trace_buffer
+#endif
+
 int head_group_size(int heads) { return heads <= 16 ? 16 : (heads <= 32 ? 32 : 64); }
 
 DecodeWorkspace decode_workspace_layout(int batch, int heads, int grid) {
@@ -1071,6 +1080,11 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
   prm.qimg = ws + w.qimg_off;
   prm.dev_err = a.dev_err;
   prm.grid = a.grid;
+#ifdef QMLA_TRACE_BUILD
+  prm.trace = g_trace_buf;
+#else
+  prm.trace = nullptr;
+#endif
   if (a.cache_kind == 4) return launch_hg<4>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
   if (a.cache_kind == 2) return launch_hg<2>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
   return launch_hg<16>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
@@ -1078,8 +1092,8 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
 
 #ifdef QMLA_TRACE_BUILD
 cudaError_t set_trace_buffer(void* buf) {
-  unsigned long long* p = static_cast<unsigned long long*>(buf);
-  return cudaMemcpyToSymbol(g_trace, &p, sizeof(p));
+  g_trace_buf = static_cast<unsigned long long*>(buf);
+  return cudaSuccess;
 }
 #endif
 
