@@ -57,7 +57,7 @@ constexpr float kLn2 = 0.6931471805599453f;
 // Optional per-CTA timeline (clock64 at pipeline events), compiled in only
 // for trace builds (-DQMLA_TRACE_BUILD); see qmla_trace_set in api.cu.
 #ifdef QMLA_TRACE_BUILD
-constexpr int kTraceCtas = 8, kTraceEvents = 96, kTraceTiles = 32;
+constexpr int kTraceCtas = 8, kTraceEvents = 128, kTraceTiles = 32;
 // The buffer pointer travels in the kernel parameters (constant bank), so an
 // event costs one clock read and one global store, no load.
 #define QMLA_TRACE(ev, tile)                                                                     \
@@ -104,9 +104,11 @@ struct __align__(16) Ctrl {
   uint32_t vote[2][4];
   alignas(16) float m_ref[64];  // read as float4
   alignas(16) float alpha[64];
+  alignas(16) float inv[64];  // 1 / l per head at a segment end, read as float4
   alignas(16) float red[4][64];
 };
-static_assert(offsetof(Ctrl, m_ref) % 16 == 0 && offsetof(Ctrl, alpha) % 16 == 0, "float4 access alignment");
+static_assert(offsetof(Ctrl, m_ref) % 16 == 0 && offsetof(Ctrl, alpha) % 16 == 0 && offsetof(Ctrl, inv) % 16 == 0,
+              "float4 access alignment");
 static_assert(sizeof(Ctrl) % 16 == 0, "Ctrl size");
 
 template <int HG>
@@ -526,6 +528,7 @@ __device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint8_t* qs
     const TileInfo ti = tile_info(sc, p);
     if (leader) QMLA_TRACE(10, it);
     if (ti.first && !(ok = wwait(&ctl.q_full, seg & 1u, ctl, kSiteMmaQFull, p.dev_err))) break;
+    if (leader && ti.first) QMLA_TRACE(110, it);
     // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576).
     if (!(ok = wwait(&ctl.tile_full, it & 1u, ctl, kSiteMmaFull, p.dev_err))) break;
     tc_fence_after();
@@ -701,6 +704,7 @@ __device__ void softmax_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& c
     if (ti.first) {
       // New segment: the reference is this tile's max.
       warp_tile_max<HG>(t_s, sl2, valid, ctl, q4, lane);
+      if (lane == 0 && q4 == 0) QMLA_TRACE(111, it);
       if (!(ok = group_sync(&ctl.grp[1], gph[1], ctl, kSiteSmMax, p.dev_err))) break;
       if (row < HG)
         ctl.m_ref[row] = fmaxf(fmaxf(ctl.red[0][row], ctl.red[1][row]), fmaxf(ctl.red[2][row], ctl.red[3][row]));
@@ -771,6 +775,7 @@ __device__ void softmax_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& c
     }
 
     if (ti.last) {
+      if (lane == 0 && q4 == 0) QMLA_TRACE(100, it);
       // Segment end: l[h] = sum of the row sums over the 128 rows; then O^T.
 #pragma unroll
       for (int c = 0; c < NC; ++c) {
@@ -783,36 +788,51 @@ __device__ void softmax_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& c
         const float tot = warp_colsum16(v, lane);
         if ((lane & 1) == 0) ctl.red[q4][c * 16 + (lane >> 1)] = tot;
       }
+      if (lane == 0 && q4 == 0) QMLA_TRACE(101, it);
       if (!(ok = group_sync(&ctl.grp[1], gph[1], ctl, kSiteSmLsum, p.dev_err))) break;
-      if (row < HG) ctl.alpha[row] = (ctl.red[0][row] + ctl.red[1][row]) + (ctl.red[2][row] + ctl.red[3][row]);
+      if (row < HG) {
+        const float l = (ctl.red[0][row] + ctl.red[1][row]) + (ctl.red[2][row] + ctl.red[3][row]);
+        ctl.alpha[row] = l;
+        ctl.inv[row] = 1.0f / l;  // one division per head; the rows below are multiplied
+      }
       if (!(ok = group_sync(&ctl.grp[2], gph[2], ctl, kSiteSmL, p.dev_err))) break;
+      if (lane == 0 && q4 == 0) QMLA_TRACE(102, it);
       if (!(ok = wwait(&ctl.pv_done, it & 1u, ctl, kSiteSmPvEpi, p.dev_err))) break;
       tc_fence_after();
+      if (lane == 0 && q4 == 0) QMLA_TRACE(103, it);
       const bool whole = (seg_j0 == 0) && (sc.t + 1 == sc.pu1);
       const int h0 = ti.hg * HG;
+      const int hn = min(HG, p.heads - h0);
       const size_t pidx = static_cast<size_t>(blockIdx.x) + sc.u;
+      // Whole segment: out = O / l (products with the per-head reciprocal);
+      // split segment: the unnormalised partial o.
+      float* const obase =
+          whole ? p.out + (static_cast<size_t>(ti.b) * p.heads + h0) * kDc : p.part_o + pidx * HG * kDc;
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         const int P = i * 128 + row;  // position in the reconstructed row
-        const int ch = (P & ~7) + Perm<CB>::at(P & 7);
+        float* const orow = obase + (P & ~7) + Perm<CB>::at(P & 7);
 #pragma unroll
         for (int c = 0; c < NC; ++c) {
           uint32_t r[16];
           tmem_ld16(t_o + i * HG + c * 16, r);
+          float f[16];
+#pragma unroll
+          for (int v4 = 0; v4 < 4; ++v4) {
+            const float4 iv = whole ? reinterpret_cast<const float4*>(ctl.inv)[c * 4 + v4] : make_float4(1.f, 1.f, 1.f, 1.f);
+            f[4 * v4] = iv.x;
+            f[4 * v4 + 1] = iv.y;
+            f[4 * v4 + 2] = iv.z;
+            f[4 * v4 + 3] = iv.w;
+          }
           tmem_ld_wait();
 #pragma unroll
           for (int jj = 0; jj < 16; ++jj) {
             const int h = c * 16 + jj;
-            if (h0 + h < p.heads) {
-              const float v = __uint_as_float(r[jj]);
-              if (whole) {
-                p.out[(static_cast<size_t>(ti.b) * p.heads + h0 + h) * kDc + ch] = v / ctl.alpha[h];
-              } else {
-                p.part_o[(pidx * HG + h) * kDc + ch] = v;
-              }
-            }
+            if (h < hn) orow[static_cast<size_t>(h) * kDc] = __uint_as_float(r[jj]) * f[jj];
           }
         }
+        if (lane == 0 && q4 == 0) QMLA_TRACE(104 + i, it);
       }
       if (row < HG && h0 + row < p.heads) {
         if (whole) {
@@ -828,6 +848,7 @@ __device__ void softmax_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& c
       if (lane == 0) {
         mbar_arrive(&ctl.o_free);
         if (q4 == 0) QMLA_TRACE(20, it);
+        if (q4 == 0) QMLA_TRACE(108, it);
       }
     }
     ++it;
