@@ -46,10 +46,9 @@ namespace {
 constexpr int kTileTokens = 128;                 // tokens per tile (M of QK)
 constexpr int kChunkBytes = kTileTokens * 128;   // 128 tokens x 64 fp16 channels
 constexpr int kNumChunks = 9;                    // 8 content chunks + RoPE-key chunk
-constexpr int kNumDqWarps = 8;
-constexpr int kSmWarp0 = kNumDqWarps;            // softmax warps 8..11 (TMEM lane quarters 0..3)
-constexpr int kMmaWarp = kNumDqWarps + 4;        // warp 12 issues MMAs and owns TMEM
-constexpr int kThreads = (kMmaWarp + 1) * 32;    // 416
+constexpr int kWorkers = 8;                      // warps 0..7: dequantise, softmax, epilogue
+constexpr int kMmaWarp = kWorkers;               // warp 8 issues MMAs and owns TMEM
+constexpr int kThreads = (kMmaWarp + 1) * 32;    // 288
 constexpr uint64_t kWaitNs = 2000000000ull;      // bound of every on-chip wait (2 s)
 constexpr float kRescaleLog2 = 8.0f;             // rescale O only above 2^8 growth
 constexpr float kLn2 = 0.6931471805599453f;
@@ -86,6 +85,7 @@ struct Params {
   float* lse;
   const int32_t* prefix;
   int32_t* prefix_w;
+  int32_t* cta_unit;  // [grid]: unit holding each CTA's first tile (written with the prefix)
   float* part_o;   // [(grid + units)][HG][512]
   float* part_ml;  // [(grid + units)][HG][2]
   uint8_t* qimg;   // [units][9][HG][128 B]: swizzled fp16 query tiles
@@ -95,13 +95,17 @@ struct Params {
 };
 
 struct __align__(16) Ctrl {
-  // tile_full: every chunk of the tile is written (one arrive per dequant warp).
-  // pv_done: the tile's PV has completed, so every chunk slot is free again.
-  uint64_t tile_full, s_full, p_full, pv_done, o_free, q_full, fin;
-  uint64_t grp[3];
+  // chunk_full[k]: chunk k of the current tile is written (one arrive per warp of its parity).
+  // slot_free[j]: PV block j (chunks 2j, 2j+1) of the previous tile has completed.
+  // pv_done: a tile's whole PV has completed: chunks 6, 7 and the P tile (chunk 8's
+  // slot) are free and O^T holds the sum through that tile.
+  uint64_t chunk_full[kNumChunks];
+  uint64_t slot_free[3];
+  uint64_t pv_done, s_full, p_full, o_free, q_full, fin;
+  uint64_t grp;  // barrier among the worker warps (one arrive per warp, reused in sequence)
   uint32_t tmem_base;
   uint32_t abort;
-  uint32_t vote[2][4];
+  uint32_t vote[2][kWorkers];
   alignas(16) float m_ref[64];  // read as float4
   alignas(16) float alpha[64];
   alignas(16) float inv[64];  // 1 / l per head at a segment end, read as float4
@@ -180,9 +184,8 @@ __device__ __forceinline__ float warp_max_f32(float v) {
 
 // Wait sites, reported in bits 8.. of the error word when a wait runs out.
 enum WaitSite : uint32_t {
-  kSiteDqEmpty = 0, kSiteMmaQFull, kSiteMmaFull, kSiteMmaPFull, kSiteMmaOFree,
-  kSiteSmSFull, kSiteSmVote, kSiteSmMax, kSiteSmFinal, kSiteSmPvRescale, kSiteSmLsum, kSiteSmL,
-  kSiteSmPvEpi, kSiteMmaFin
+  kSiteDqSlot = 0, kSiteMmaQFull, kSiteMmaChunk, kSiteMmaPFull, kSiteMmaOFree,
+  kSiteSmSFull, kSiteGrp, kSitePvEpi, kSiteMmaFin
 };
 
 // Marks the CTA aborted; a wait that ran out (rather than saw the abort)
@@ -210,12 +213,13 @@ __device__ __forceinline__ bool wwait(uint64_t* bar, uint32_t parity, Ctrl& c, u
   if (r == 0) wait_ok(r, site, c, dev_err);
   return all_ok;
 }
-// Barrier among the four softmax warps (one arrive per warp), bounded.
-__device__ __forceinline__ bool group_sync(uint64_t* bar, uint32_t& phase, Ctrl& c, uint32_t site,
-                                           uint32_t* dev_err) {
+// Barrier among the worker warps (one arrive per warp), bounded. Every worker
+// passes the same sequence of these, so one mbarrier serves them all: a warp
+// cannot arrive for phase n + 2 before every warp has arrived for n + 1.
+__device__ __forceinline__ bool group_sync(Ctrl& c, uint32_t& phase, uint32_t* dev_err) {
   __syncwarp();
-  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
-  const bool ok = wwait(bar, phase & 1u, c, site, dev_err);
+  if ((threadIdx.x & 31) == 0) mbar_arrive(&c.grp);
+  const bool ok = wwait(&c.grp, phase & 1u, c, kSiteGrp, dev_err);
   ++phase;
   return ok;
 }
@@ -225,7 +229,8 @@ struct Sched {
   const int32_t* prefix;
   int t0, t1, t, u, pu0, pu1;
   int units;
-  __device__ void init(const int32_t* pf, int units_, int cta, int grid) {
+  // cu[cta] is the unit holding tile t0 (found once by the prep kernel).
+  __device__ void init(const int32_t* pf, const int32_t* cu, int units_, int cta, int grid) {
     prefix = pf;
     units = units_;
     const int T = pf[units];
@@ -235,12 +240,7 @@ struct Sched {
     u = 0;
     pu0 = pu1 = 0;
     if (t0 >= t1) return;
-    int lo = 0, hi = units_;  // prefix[lo] <= t0 < prefix[hi]
-    while (hi - lo > 1) {
-      const int mid = (lo + hi) >> 1;
-      if (pf[mid] <= t0) lo = mid; else hi = mid;
-    }
-    u = lo;
+    u = cu[cta];
     pu0 = pf[u];
     pu1 = pf[u + 1];
   }
@@ -404,90 +404,396 @@ __device__ __forceinline__ void query_piece(const Params& p, uint8_t* img, int b
   *reinterpret_cast<uint4*>(img + k * HG * 128 + swz_off(h, i, 128)) = o;
 }
 
-template <int CB, int HG>
-__device__ void dequant_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ctl, int warp, int lane) {
-  const int row = (warp & 3) * 32 + lane;  // token row of the tile
-  const int par = warp >> 2;               // this warp handles chunks k = par, par+2, ...
-  const int slot = row & 63;
-  uint32_t it = 0;
-  Fetch f[5];
-  TileInfo ti;
-  bool ok = true;
-  if (sc.valid()) {
-    ti = tile_info(sc, p);
-    if constexpr (CB != 16) {
-      bool valid;
-      const uint8_t* blk = row_block<CB>(p, ti, row, valid);
+// ------------------------------------------------------------ worker warps
+// Eight worker warps dequantise each tile, compute its softmax and write the
+// segment results. Warp w owns token rows 32 (w & 3) .. 32 (w & 3) + 31 (its
+// TMEM lane quarter), dequantises the chunks of parity w >> 2 and, in the
+// softmax and epilogue, the heads [(w >> 2) HG/2, (w >> 2 + 1) HG/2).
+template <int HG>
+struct Cols {
+  static constexpr int kPerWarp = HG / 2;       // heads per worker warp
+  static constexpr int kW = HG >= 32 ? 16 : 8;  // TMEM columns per load
+  static constexpr int kN = kPerWarp / kW;      // loads per column set
+  static_assert(kN * kW == kPerWarp, "column split");
+};
+
+// The slot of chunk k is freed by PV block k / 2 of the previous tile; the
+// RoPE chunk 8 holds that tile's P and is freed by the whole PV.
+__device__ __forceinline__ uint64_t* slot_bar(Ctrl& c, int k) { return k < 6 ? &c.slot_free[k >> 1] : &c.pv_done; }
+
+// Sum over the warp's 32 lanes of each of W values; lane l returns the total
+// of element l >> 1 (W = 16) or l >> 2 (W = 8), by recursive halving.
+template <int W>
+__device__ __forceinline__ float warp_colsum(float (&v)[W], int lane) {
 #pragma unroll
-      for (int kc = 0; kc < 5; ++kc) {
+  for (int s = 16, n = W / 2; n >= 1; s >>= 1, n >>= 1) {
+    const bool hi = (lane & s) != 0;
+#pragma unroll
+    for (int i = 0; i < n; ++i) {
+      const float send = hi ? v[i] : v[i + n];
+      const float keep = hi ? v[i + n] : v[i];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, s);
+    }
+  }
+  float t = v[0];
+  constexpr int kRest = W == 16 ? 1 : 2;  // lanes still holding partial sums of one element
+#pragma unroll
+  for (int s = kRest; s >= 1; s >>= 1) t += __shfl_xor_sync(0xffffffffu, t, s);
+  return t;
+}
+
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Tile max of the scaled scores of this warp's heads over its 32 rows into red_q[h].
+template <int HG>
+__device__ __forceinline__ void warp_tile_max(uint32_t t_s, float sl2, bool valid, float* red_q, int lane) {
+  using C = Cols<HG>;
+#pragma unroll
+  for (int c = 0; c < C::kN; ++c) {
+    uint32_t r[C::kW];
+    tmem_ld(t_s + c * C::kW, r);
+    tmem_ld_wait();
+#pragma unroll
+    for (int jj = 0; jj < C::kW; ++jj) {
+      const float x = valid ? __uint_as_float(r[jj]) * sl2 : -INFINITY;
+      const float mx = warp_max_f32(x);
+      if (lane == jj) red_q[c * C::kW + jj] = mx;
+    }
+  }
+}
+
+// P^T[t, h] = 2^(S * scale * log2e - m_ref[h]) in fp16 for this warp's heads,
+// into row t of the P tile and into pk; returns whether a weight exceeds 2^8.
+template <int HG>
+__device__ __forceinline__ bool compute_p(uint32_t t_s, const float* mr, float sl2, bool valid, uint32_t ptile,
+                                          int row, int piece0, uint32_t (&pk)[Cols<HG>::kPerWarp / 2]) {
+  using C = Cols<HG>;
+  constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
+  bool over = false;
+#pragma unroll
+  for (int c = 0; c < C::kN; ++c) {
+    uint32_t r[C::kW];
+    tmem_ld(t_s + c * C::kW, r);
+    float m[C::kW];
+#pragma unroll
+    for (int v4 = 0; v4 < C::kW / 4; ++v4) {
+      const float4 mv = reinterpret_cast<const float4*>(mr)[c * (C::kW / 4) + v4];
+      m[4 * v4] = mv.x;
+      m[4 * v4 + 1] = mv.y;
+      m[4 * v4 + 2] = mv.z;
+      m[4 * v4 + 3] = mv.w;
+    }
+    tmem_ld_wait();
+#pragma unroll
+    for (int jj = 0; jj < C::kW; jj += 2) {
+      const float x0 = __uint_as_float(r[jj]) * sl2 - m[jj];
+      const float x1 = __uint_as_float(r[jj + 1]) * sl2 - m[jj + 1];
+      over |= valid && (fmaxf(x0, x1) > kRescaleLog2);
+      pk[c * (C::kW / 2) + (jj >> 1)] = valid ? pack_h2(ex2_approx(x0), ex2_approx(x1)) : 0u;
+    }
+#pragma unroll
+    for (int pc = 0; pc < C::kW / 8; ++pc) {
+      const uint32_t* w = &pk[c * (C::kW / 2) + 4 * pc];
+      sts_v4(ptile + swz_off(row, piece0 + c * (C::kW / 8) + pc, kRB), w[0], w[1], w[2], w[3]);
+    }
+  }
+  return over;
+}
+
+// What a segment end needs once its last PV has completed.
+struct SegEnd {
+  int b, hg;
+  bool whole;   // the segment is the whole unit: write out / lse, else a partial
+  size_t pidx;  // partial slot (CTA index + unit)
+};
+
+// Segment end: l[h] = sum of the row sums, then out = O / l (or the partial
+// o, m, l) for this warp's heads, then release O^T to the next segment.
+template <int CB, int HG>
+__device__ bool epilogue(const Params& p, const SegEnd& e, Ctrl& ctl, uint32_t tmem, uint32_t& gph, int warp,
+                         int lane) {
+  using C = Cols<HG>;
+  const int q4 = warp & 3, half = warp >> 2, row = q4 * 32 + lane, cb0 = half * C::kPerWarp;
+  const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
+  const uint32_t t_l = tmem + 5 * HG + cb0 + lane_off;
+  const uint32_t t_o = tmem + cb0 + lane_off;
+#pragma unroll
+  for (int c = 0; c < C::kN; ++c) {
+    uint32_t r[C::kW];
+    tmem_ld(t_l + c * C::kW, r);
+    tmem_ld_wait();
+    float v[C::kW];
+#pragma unroll
+    for (int jj = 0; jj < C::kW; ++jj) v[jj] = __uint_as_float(r[jj]);
+    const float tot = warp_colsum<C::kW>(v, lane);
+    constexpr int kSh = C::kW == 16 ? 1 : 2;
+    if ((lane & ((1 << kSh) - 1)) == 0) ctl.red[q4][cb0 + c * C::kW + (lane >> kSh)] = tot;
+  }
+  if (!group_sync(ctl, gph, p.dev_err)) return false;
+  const int tid = threadIdx.x;  // 0 .. 255 over the worker warps
+  if (tid < HG) {
+    const float l = (ctl.red[0][tid] + ctl.red[1][tid]) + (ctl.red[2][tid] + ctl.red[3][tid]);
+    ctl.alpha[tid] = l;
+    ctl.inv[tid] = 1.0f / l;  // one division per head; the rows below are multiplied
+  }
+  if (!group_sync(ctl, gph, p.dev_err)) return false;
+  const int h0 = e.hg * HG;
+  const int hn = min(HG, p.heads - h0);
+  float* const obase =
+      e.whole ? p.out + (static_cast<size_t>(e.b) * p.heads + h0) * kDc : p.part_o + e.pidx * HG * kDc;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int P = i * 128 + row;  // position in the reconstructed row
+    float* const orow = obase + (P & ~7) + Perm<CB>::at(P & 7);
+#pragma unroll
+    for (int c = 0; c < C::kN; ++c) {
+      uint32_t r[C::kW];
+      tmem_ld(t_o + i * HG + c * C::kW, r);
+      float f[C::kW];
+#pragma unroll
+      for (int v4 = 0; v4 < C::kW / 4; ++v4) {
+        const float4 iv = e.whole ? reinterpret_cast<const float4*>(ctl.inv + cb0)[c * (C::kW / 4) + v4]
+                                  : make_float4(1.f, 1.f, 1.f, 1.f);
+        f[4 * v4] = iv.x;
+        f[4 * v4 + 1] = iv.y;
+        f[4 * v4 + 2] = iv.z;
+        f[4 * v4 + 3] = iv.w;
+      }
+      tmem_ld_wait();
+#pragma unroll
+      for (int jj = 0; jj < C::kW; ++jj) {
+        const int h = cb0 + c * C::kW + jj;
+        if (h < hn) orow[static_cast<size_t>(h) * kDc] = __uint_as_float(r[jj]) * f[jj];
+      }
+    }
+  }
+  if (tid < HG && h0 + tid < p.heads) {
+    if (e.whole) {
+      if (p.lse != nullptr)
+        p.lse[static_cast<size_t>(e.b) * p.heads + h0 + tid] = (ctl.m_ref[tid] + log2f(ctl.alpha[tid])) * kLn2;
+    } else {
+      p.part_ml[(e.pidx * HG + tid) * 2 + 0] = ctl.m_ref[tid];
+      p.part_ml[(e.pidx * HG + tid) * 2 + 1] = ctl.alpha[tid];
+    }
+  }
+  tc_fence_before();
+  __syncwarp();
+  if (lane == 0) mbar_arrive(&ctl.o_free);
+  return true;
+}
+
+template <int CB, int HG>
+__device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ctl, uint32_t tmem, int warp,
+                            int lane) {
+  using C = Cols<HG>;
+  const int q4 = warp & 3;
+  const int par = warp >> 2;  // dequantised chunks k = par, par + 2, ...; heads half `par`
+  const int row = q4 * 32 + lane;
+  const int slot = row & 63;
+  const int cb0 = par * C::kPerWarp;
+  const int piece0 = cb0 / 8;
+  const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
+  const uint32_t t_s = tmem + 4 * HG + cb0 + lane_off;
+  const uint32_t t_o = tmem + cb0 + lane_off;
+  const uint32_t t_l = tmem + 5 * HG + cb0 + lane_off;
+  const uint32_t ptile = chunks + 8 * kChunkBytes;
+  const float sl2 = p.scale_log2;
+  constexpr int kMyChunks = 5;  // chunks per parity, rounded up (parity 1 has 4)
+  uint32_t it = 0, gph = 0;
+  int seg_j0 = 0;
+  bool ok = true;
+  bool pending = false;  // the previous tile ended a segment whose epilogue is still due
+  SegEnd pend{};
+
+  // Packed rows of the tile about to be dequantised (INT4/INT2), fetched a tile ahead.
+  Fetch f[kMyChunks];
+  // BF16 cache: one chunk row (8 x 16 B) of look-ahead.
+  uint4 cur[CB == 16 ? 8 : 1];
+  auto fetch_tile = [&](const Sched& s) {
+    bool valid = false;
+    const TileInfo tf = tile_info(s, p);
+    const uint8_t* blk = row_block<CB>(p, tf, row, valid);
+    if constexpr (CB != 16) {
+#pragma unroll
+      for (int kc = 0; kc < kMyChunks; ++kc) {
         const int k = 2 * kc + par;
         if (k < kNumChunks) f[kc] = fetch_chunk<CB>(blk, valid, k, slot);
       }
     }
-  }
-  while (ok && sc.valid()) {
-    // Phased schedule: the tile is written while the tensor pipe is idle
-    // (after the previous tile's PV), because generic shared-memory stores
-    // are starved while the tensor core streams its operands.
-    if (!wwait(&ctl.pv_done, (it & 1u) ^ 1u, ctl, kSiteDqEmpty, p.dev_err)) {
-      ok = false;
-      break;
-    }
-    if (lane == 0 && warp == 0) QMLA_TRACE(0, it);
-    if (lane == 0) QMLA_TRACE(40 + warp, it);
+    return blk;
+  };
+  const uint8_t* blk_cur = nullptr;
+  bool valid_cur = false;
+  if (sc.valid()) {
+    blk_cur = fetch_tile(sc);
+    valid_cur = blk_cur != nullptr;
     if constexpr (CB == 16) {
-      bool valid16 = false;
-      const uint8_t* blk16 = row_block<CB>(p, ti, row, valid16);
-      uint4 v[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i)
-        v[i] = valid16 ? ldg_nc_v4(blk16 + slot * (kDqk * 2) + par * 128 + i * 16) : make_uint4(0, 0, 0, 0);
-#pragma unroll
-      for (int kc = 0; kc < 5; ++kc) {
-        const int k = 2 * kc + par;
-        if (k >= kNumChunks) break;
-        uint4 cur[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) cur[i] = v[i];
-        if (k + 2 < kNumChunks) {
-#pragma unroll
-          for (int i = 0; i < 8; ++i)
-            v[i] = valid16 ? ldg_nc_v4(blk16 + slot * (kDqk * 2) + (k + 2) * 128 + i * 16) : make_uint4(0, 0, 0, 0);
-        }
-        store_row_bf16(chunks + k * kChunkBytes, row, cur, valid16);
-      }
-    } else {
-#pragma unroll
-      for (int kc = 0; kc < 5; ++kc) {
-        const int k = 2 * kc + par;
-        if (k >= kNumChunks) break;
-        store_row<CB>(chunks + k * kChunkBytes, row, f[kc], CB == 4 || k == 8);
-        if (lane == 0) QMLA_TRACE(48 + warp * 5 + kc, it);
-      }
-    }
-    fence_proxy_async_smem();
-    __syncwarp();
-    if (lane == 0) {
-      mbar_arrive(&ctl.tile_full);
-      QMLA_TRACE(32 + warp, it);
-    }
-    if (!ok) break;
-    ++it;
-    sc.next();
-    if (sc.valid()) {
-      ti = tile_info(sc, p);
-      if constexpr (CB != 16) {
-        bool valid;
-        const uint8_t* blk = row_block<CB>(p, ti, row, valid);
-#pragma unroll
-        for (int kc = 0; kc < 5; ++kc) {
-          const int k = 2 * kc + par;
-          if (k < kNumChunks) f[kc] = fetch_chunk<CB>(blk, valid, k, slot);
-        }
-      }
+        cur[i] = valid_cur ? ldg_nc_v4(blk_cur + slot * (kDqk * 2) + par * 128 + i * 16) : make_uint4(0, 0, 0, 0);
     }
   }
-  if (!ok) set_abort(ctl, p.dev_err);
+
+  for (; ok && sc.valid(); sc.next()) {
+    const TileInfo ti = tile_info(sc, p);
+    if (ti.first) seg_j0 = ti.j;
+    const bool valid = row < ti.ntok;
+    Sched nx = sc;
+    nx.next();
+    const bool has_next = nx.valid();
+    bool valid_nx = false;
+    const uint8_t* blk_nx = nullptr;
+    if (has_next) {
+      const TileInfo tn = tile_info(nx, p);
+      blk_nx = row_block<CB>(p, tn, row, valid_nx);
+    }
+    if (lane == 0 && warp == 0) QMLA_TRACE(0, it);
+
+    // ---- dequantise this tile, chunk by chunk as the previous PV frees the slots
+#pragma unroll
+    for (int kc = 0; kc < kMyChunks; ++kc) {
+      const int k = 2 * kc + par;
+      if (k >= kNumChunks) break;
+      if (!(ok = wwait(slot_bar(ctl, k), (it & 1u) ^ 1u, ctl, kSiteDqSlot, p.dev_err))) break;
+      if constexpr (CB == 16) {
+        uint4 nxt[8];
+        const int kn = k + 2;
+        if (kn < kNumChunks) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            nxt[i] = valid_cur ? ldg_nc_v4(blk_cur + slot * (kDqk * 2) + kn * 128 + i * 16) : make_uint4(0, 0, 0, 0);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            nxt[i] = valid_nx ? ldg_nc_v4(blk_nx + slot * (kDqk * 2) + par * 128 + i * 16) : make_uint4(0, 0, 0, 0);
+        }
+        store_row_bf16(chunks + k * kChunkBytes, row, cur, valid_cur);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) cur[i] = nxt[i];
+      } else {
+        store_row<CB>(chunks + k * kChunkBytes, row, f[kc], CB == 4 || k == 8);
+        f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);  // the next tile's rows of this chunk
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.chunk_full[k]);
+    }
+    if (!ok) break;
+    if (lane == 0) QMLA_TRACE(32 + warp, it);
+    blk_cur = blk_nx;
+    valid_cur = valid_nx;
+
+    // ---- the previous segment's results (its last PV completed: chunks 6..8 were waited for)
+    if (pending) {
+      tc_fence_after();
+      if (!(ok = epilogue<CB, HG>(p, pend, ctl, tmem, gph, warp, lane))) break;
+      pending = false;
+      if (lane == 0 && warp == 0) QMLA_TRACE(20, it);
+    }
+
+    // ---- softmax of this tile
+    if (!(ok = wwait(&ctl.s_full, it & 1u, ctl, kSiteSmSFull, p.dev_err))) break;
+    tc_fence_after();
+    if (lane == 0 && warp == 0) QMLA_TRACE(16, it);
+    if (ti.first) {
+      // New segment: the reference is this tile's max.
+      warp_tile_max<HG>(t_s, sl2, valid, &ctl.red[q4][cb0], lane);
+      if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
+      if (threadIdx.x < HG) {
+        const int h = threadIdx.x;
+        ctl.m_ref[h] = fmaxf(fmaxf(ctl.red[0][h], ctl.red[1][h]), fmaxf(ctl.red[2][h], ctl.red[3][h]));
+      }
+      if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
+    }
+    uint32_t pk[C::kPerWarp / 2];
+    const bool over = compute_p<HG>(t_s, ctl.m_ref + cb0, sl2, valid, ptile, row, piece0, pk);
+    uint32_t* vote = ctl.vote[it & 1u];
+    const uint32_t any = __any_sync(0xffffffffu, over);
+    if (lane == 0) vote[warp] = any;
+    if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
+    if (lane == 0 && warp == 0) QMLA_TRACE(17, it);
+    uint32_t anyv = 0;
+#pragma unroll
+    for (int w = 0; w < kWorkers; ++w) anyv |= vote[w];
+    if (anyv != 0u) {
+      // Raise the reference to the running max; O and the row sums were
+      // accumulated against the old one and are scaled by alpha = 2^(m_old - m_new).
+      // The previous PV has completed (its slots were waited for above).
+      warp_tile_max<HG>(t_s, sl2, valid, &ctl.red[q4][cb0], lane);
+      if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
+      if (threadIdx.x < HG) {
+        const int h = threadIdx.x;
+        const float mt = fmaxf(fmaxf(ctl.red[0][h], ctl.red[1][h]), fmaxf(ctl.red[2][h], ctl.red[3][h]));
+        const float mo = ctl.m_ref[h];
+        const float mn = fmaxf(mo, mt);
+        ctl.alpha[h] = exp2f(mo - mn);
+        ctl.m_ref[h] = mn;
+      }
+      if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
+      if (!ti.first) {
+#pragma unroll
+        for (int i = 0; i < 5; ++i) {  // O^T blocks 0..3 and the row sums (column block 5)
+          const uint32_t col = i < 4 ? i * HG : 5 * HG;
+#pragma unroll
+          for (int c = 0; c < C::kN; ++c) {
+            uint32_t r[C::kW];
+            tmem_ld(t_o + col + c * C::kW, r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int jj = 0; jj < C::kW; ++jj)
+              r[jj] = __float_as_uint(__uint_as_float(r[jj]) * ctl.alpha[cb0 + c * C::kW + jj]);
+            tmem_st(t_o + col + c * C::kW, r);
+          }
+        }
+        tmem_st_wait();
+      }
+      compute_p<HG>(t_s, ctl.m_ref + cb0, sl2, valid, ptile, row, piece0, pk);
+    }
+    // Row sums of the fp16 weights the PV MMA multiplies with.
+#pragma unroll
+    for (int c = 0; c < C::kN; ++c) {
+      uint32_t r[C::kW];
+      if (!ti.first) {
+        tmem_ld(t_l + c * C::kW, r);
+        tmem_ld_wait();
+      }
+#pragma unroll
+      for (int jj = 0; jj < C::kW; jj += 2) {
+        const float2 pf = __half22float2(*reinterpret_cast<const __half2*>(&pk[c * (C::kW / 2) + (jj >> 1)]));
+        r[jj] = __float_as_uint(ti.first ? pf.x : __uint_as_float(r[jj]) + pf.x);
+        r[jj + 1] = __float_as_uint(ti.first ? pf.y : __uint_as_float(r[jj + 1]) + pf.y);
+      }
+      tmem_st(t_l + c * C::kW, r);
+    }
+    tmem_st_wait();
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) {
+      mbar_arrive(&ctl.p_full);
+      if (warp == 0) QMLA_TRACE(19, it);
+    }
+    if (ti.last) {
+      pending = true;
+      pend.b = ti.b;
+      pend.hg = ti.hg;
+      pend.whole = (seg_j0 == 0) && (sc.t + 1 == sc.pu1);
+      pend.pidx = static_cast<size_t>(blockIdx.x) + sc.u;
+    }
+    ++it;
+  }
+  // The last segment's results once its PV has completed.
+  if (ok && pending) {
+    if ((ok = wwait(&ctl.pv_done, (it - 1) & 1u, ctl, kSitePvEpi, p.dev_err))) {
+      tc_fence_after();
+      ok = epilogue<CB, HG>(p, pend, ctl, tmem, gph, warp, lane);
+    }
+  }
+  if (!ok && lane == 0) set_abort(ctl, p.dev_err);
 }
 
 // ------------------------------------------------------------ MMA warp
@@ -504,8 +810,10 @@ __device__ __forceinline__ void issue_query(const Params& p, int unit, uint8_t* 
 
 // The MMA warp walks the schedule and waits on every lane; one elected lane
 // issues the MMAs, the commits (a commit tracks the MMAs issued by the
-// committing thread) and the query copies. Descriptors are advanced by adding
-// (byte offset >> 4) to their start-address field.
+// committing thread) and the query copies. QK starts on each chunk as soon
+// as it is written; PV commits after each 128-channel block so that the next
+// tile's dequantisation can refill those slots. Descriptors are advanced by
+// adding (byte offset >> 4) to their start-address field.
 template <int HG>
 __device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint8_t* qsmem, Ctrl& ctl,
                          uint32_t tmem, int lane) {
@@ -526,16 +834,14 @@ __device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint8_t* qs
   if (sc.valid() && leader) issue_query<HG>(p, sc.u, qsmem, ctl);
   for (; ok && sc.valid(); sc.next()) {
     const TileInfo ti = tile_info(sc, p);
-    if (leader) QMLA_TRACE(10, it);
     if (ti.first && !(ok = wwait(&ctl.q_full, seg & 1u, ctl, kSiteMmaQFull, p.dev_err))) break;
-    if (leader && ti.first) QMLA_TRACE(110, it);
-    // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576).
-    if (!(ok = wwait(&ctl.tile_full, it & 1u, ctl, kSiteMmaFull, p.dev_err))) break;
-    tc_fence_after();
-    if (leader) {
-      QMLA_TRACE(11, it);
+    // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576), chunk by chunk.
 #pragma unroll 1
-      for (int k = 0; k < kNumChunks; ++k) {
+    for (int k = 0; k < kNumChunks; ++k) {
+      if (!(ok = wwait(&ctl.chunk_full[k], it & 1u, ctl, kSiteMmaChunk, p.dev_err))) break;
+      tc_fence_after();
+      if (leader) {
+        if (k == 0) QMLA_TRACE(11, it);
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk) {
           const uint64_t ad = qk_a0 + static_cast<uint64_t>((k * kChunkBytes + kk * 32) >> 4);
@@ -543,6 +849,10 @@ __device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint8_t* qs
           umma_f16_ss(t_s, ad, bd, kIdQK, (k | kk) != 0 ? 1u : 0u);
         }
       }
+      __syncwarp();
+    }
+    if (!ok) break;
+    if (leader) {
       umma_commit(&ctl.s_full);
       QMLA_TRACE(12, it);
     }
@@ -570,8 +880,8 @@ __device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint8_t* qs
           const uint64_t bd = pv_b0 + static_cast<uint64_t>((kk * 2 * kSboP) >> 4);
           umma_f16_ss(tmem + i * HG, ad, bd, kIdPV, (ti.first && kk == 0) ? 0u : 1u);
         }
+        umma_commit(i < 3 ? &ctl.slot_free[i] : &ctl.pv_done);
       }
-      umma_commit(&ctl.pv_done);
       QMLA_TRACE(15, it);
     }
     __syncwarp();
@@ -579,281 +889,12 @@ __device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint8_t* qs
     if (ti.last) ++seg;
   }
   if (!ok && leader) set_abort(ctl, p.dev_err);
-  // Every MMA and copy must have landed before TMEM and shared memory are released.
-  // This wait ignores the abort flag: TMEM may only be released once they have.
+  // Every MMA and copy must have landed before TMEM and shared memory are
+  // released; this wait ignores the abort flag.
   if (leader) umma_commit(&ctl.fin);
   __syncwarp();
   wait_ok(mbar_wait(&ctl.fin, 0, kWaitNs, nullptr), kSiteMmaFin, ctl, p.dev_err);
   __syncwarp();
-}
-
-// Column sums of a warp: v[j] summed over the 32 lanes for j = 0..15 by
-// recursive halving (16 shuffles); lane l ends with the total of element l >> 1.
-__device__ __forceinline__ float warp_colsum16(float (&v)[16], int lane) {
-  const bool b4 = lane & 16, b3 = lane & 8, b2 = lane & 4, b1 = lane & 2;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const float send = b4 ? v[i] : v[i + 8];
-    const float keep = b4 ? v[i + 8] : v[i];
-    v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
-  }
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float send = b3 ? v[i] : v[i + 4];
-    const float keep = b3 ? v[i + 4] : v[i];
-    v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
-  }
-#pragma unroll
-  for (int i = 0; i < 2; ++i) {
-    const float send = b2 ? v[i] : v[i + 2];
-    const float keep = b2 ? v[i + 2] : v[i];
-    v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
-  }
-  {
-    const float send = b1 ? v[0] : v[1];
-    const float keep = b1 ? v[1] : v[0];
-    v[0] = keep + __shfl_xor_sync(0xffffffffu, send, 2);
-  }
-  return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 1);
-}
-
-// --------------------------------------------------------- softmax warps
-__device__ __forceinline__ float ex2_approx(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
-// Tile max of the scaled scores per head into red[q4][h] (one warp's 32 rows).
-template <int HG>
-__device__ __forceinline__ void warp_tile_max(uint32_t t_s, float sl2, bool valid, Ctrl& ctl, int q4, int lane) {
-#pragma unroll
-  for (int c = 0; c < HG / 16; ++c) {
-    uint32_t r[16];
-    tmem_ld16(t_s + c * 16, r);
-    tmem_ld_wait();
-#pragma unroll
-    for (int jj = 0; jj < 16; ++jj) {
-      const float x = valid ? __uint_as_float(r[jj]) * sl2 : -INFINITY;
-      const float mx = warp_max_f32(x);
-      if (lane == jj) ctl.red[q4][c * 16 + jj] = mx;
-    }
-  }
-}
-
-// P^T[t, h] = 2^(S * scale * log2e - m_ref[h]) as fp16 into the P tile (row t)
-// and into pk; returns whether any of this thread's weights exceeds 2^8.
-template <int HG>
-__device__ __forceinline__ bool compute_p(uint32_t t_s, const float* m_ref, float sl2, bool valid, uint32_t ptile,
-                                          int row, uint32_t (&pk)[HG / 16][8]) {
-  constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
-  bool over = false;
-#pragma unroll
-  for (int c = 0; c < HG / 16; ++c) {
-    uint32_t r[16];
-    tmem_ld16(t_s + c * 16, r);
-    float m[16];
-#pragma unroll
-    for (int v4 = 0; v4 < 4; ++v4) {
-      const float4 mv = reinterpret_cast<const float4*>(m_ref)[c * 4 + v4];
-      m[4 * v4] = mv.x;
-      m[4 * v4 + 1] = mv.y;
-      m[4 * v4 + 2] = mv.z;
-      m[4 * v4 + 3] = mv.w;
-    }
-    tmem_ld_wait();
-#pragma unroll
-    for (int jj = 0; jj < 16; jj += 2) {
-      const float x0 = __uint_as_float(r[jj]) * sl2 - m[jj];
-      const float x1 = __uint_as_float(r[jj + 1]) * sl2 - m[jj + 1];
-      over |= valid && (fmaxf(x0, x1) > kRescaleLog2);
-      pk[c][jj >> 1] = valid ? pack_h2(ex2_approx(x0), ex2_approx(x1)) : 0u;
-    }
-    sts_v4(ptile + swz_off(row, 2 * c, kRB), pk[c][0], pk[c][1], pk[c][2], pk[c][3]);
-    sts_v4(ptile + swz_off(row, 2 * c + 1, kRB), pk[c][4], pk[c][5], pk[c][6], pk[c][7]);
-  }
-  return over;
-}
-
-// Softmax warps (TMEM lane quarter q4 = token rows 32 q4 .. 32 q4 + 31). Per
-// tile: P against the per-head reference max; only when a weight would exceed
-// 2^8 is the reference raised (O and the row sums rescaled, P recomputed).
-// The row sums of P live in TMEM columns [5 HG, 6 HG), one per head and row.
-template <int CB, int HG>
-__device__ void softmax_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ctl, uint32_t tmem,
-                             int warp, int lane) {
-  constexpr int NC = HG / 16;
-  const int q4 = warp & 3;
-  const int row = q4 * 32 + lane;
-  const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
-  const uint32_t t_s = tmem + 4 * HG + lane_off;
-  const uint32_t t_o = tmem + lane_off;
-  const uint32_t t_l = tmem + 5 * HG + lane_off;
-  const uint32_t ptile = chunks + 8 * kChunkBytes;
-  const float sl2 = p.scale_log2;
-  uint32_t it = 0, gph[3] = {0, 0, 0};
-  int seg_j0 = 0;
-  bool ok = true;
-  for (; ok && sc.valid(); sc.next()) {
-    const TileInfo ti = tile_info(sc, p);
-    if (ti.first) seg_j0 = ti.j;
-    const bool valid = row < ti.ntok;
-    if (!(ok = wwait(&ctl.s_full, it & 1u, ctl, kSiteSmSFull, p.dev_err))) break;
-    tc_fence_after();
-    if (lane == 0 && q4 == 0) QMLA_TRACE(16, it);
-    if (ti.first) {
-      // New segment: the reference is this tile's max.
-      warp_tile_max<HG>(t_s, sl2, valid, ctl, q4, lane);
-      if (lane == 0 && q4 == 0) QMLA_TRACE(111, it);
-      if (!(ok = group_sync(&ctl.grp[1], gph[1], ctl, kSiteSmMax, p.dev_err))) break;
-      if (row < HG)
-        ctl.m_ref[row] = fmaxf(fmaxf(ctl.red[0][row], ctl.red[1][row]), fmaxf(ctl.red[2][row], ctl.red[3][row]));
-      if (!(ok = group_sync(&ctl.grp[2], gph[2], ctl, kSiteSmFinal, p.dev_err))) break;
-    }
-    uint32_t pk[NC][8];
-    const bool over = compute_p<HG>(t_s, ctl.m_ref, sl2, valid, ptile, row, pk);
-    uint32_t* vote = ctl.vote[it & 1u];
-    const uint32_t any = __any_sync(0xffffffffu, over);
-    if (lane == 0) vote[q4] = any;
-    if (!(ok = group_sync(&ctl.grp[0], gph[0], ctl, kSiteSmVote, p.dev_err))) break;
-    if (lane == 0 && q4 == 0) QMLA_TRACE(17, it);
-    if ((vote[0] | vote[1] | vote[2] | vote[3]) != 0u) {
-      // Raise the reference to the running max; O and the row sums were
-      // accumulated against the old one and are scaled by alpha = 2^(m_old - m_new).
-      warp_tile_max<HG>(t_s, sl2, valid, ctl, q4, lane);
-      if (!(ok = group_sync(&ctl.grp[1], gph[1], ctl, kSiteSmMax, p.dev_err))) break;
-      if (row < HG) {
-        const float mt = fmaxf(fmaxf(ctl.red[0][row], ctl.red[1][row]), fmaxf(ctl.red[2][row], ctl.red[3][row]));
-        const float mo = ctl.m_ref[row];
-        const float mn = fmaxf(mo, mt);
-        ctl.alpha[row] = exp2f(mo - mn);
-        ctl.m_ref[row] = mn;
-      }
-      if (!(ok = group_sync(&ctl.grp[2], gph[2], ctl, kSiteSmFinal, p.dev_err))) break;
-      if (!(ok = wwait(&ctl.pv_done, (it - 1) & 1u, ctl, kSiteSmPvRescale, p.dev_err))) break;
-      tc_fence_after();
-#pragma unroll
-      for (int i = 0; i < 5; ++i) {  // O^T chunks 0..3 and the row sums (column block 5)
-        const uint32_t col = i < 4 ? i * HG : 5 * HG;
-#pragma unroll
-        for (int c = 0; c < NC; ++c) {
-          uint32_t r[16];
-          tmem_ld16(t_o + col + c * 16, r);
-          tmem_ld_wait();
-#pragma unroll
-          for (int jj = 0; jj < 16; ++jj) r[jj] = __float_as_uint(__uint_as_float(r[jj]) * ctl.alpha[c * 16 + jj]);
-          tmem_st16(t_o + col + c * 16, r);
-        }
-      }
-      tmem_st_wait();
-      compute_p<HG>(t_s, ctl.m_ref, sl2, valid, ptile, row, pk);
-      if (lane == 0 && q4 == 0) QMLA_TRACE(18, it);
-    }
-    // Row sums of the fp16 weights the PV MMA multiplies with.
-#pragma unroll
-    for (int c = 0; c < NC; ++c) {
-      uint32_t r[16];
-      if (!ti.first) {
-        tmem_ld16(t_l + c * 16, r);
-        tmem_ld_wait();
-      }
-#pragma unroll
-      for (int jj = 0; jj < 16; jj += 2) {
-        const float2 pf = __half22float2(*reinterpret_cast<const __half2*>(&pk[c][jj >> 1]));
-        r[jj] = __float_as_uint(ti.first ? pf.x : __uint_as_float(r[jj]) + pf.x);
-        r[jj + 1] = __float_as_uint(ti.first ? pf.y : __uint_as_float(r[jj + 1]) + pf.y);
-      }
-      tmem_st16(t_l + c * 16, r);
-    }
-    tmem_st_wait();
-    fence_proxy_async_smem();
-    tc_fence_before();
-    __syncwarp();
-    if (lane == 0) {
-      mbar_arrive(&ctl.p_full);
-      if (q4 == 0) QMLA_TRACE(19, it);
-    }
-
-    if (ti.last) {
-      if (lane == 0 && q4 == 0) QMLA_TRACE(100, it);
-      // Segment end: l[h] = sum of the row sums over the 128 rows; then O^T.
-#pragma unroll
-      for (int c = 0; c < NC; ++c) {
-        uint32_t r[16];
-        tmem_ld16(t_l + c * 16, r);
-        tmem_ld_wait();
-        float v[16];
-#pragma unroll
-        for (int jj = 0; jj < 16; ++jj) v[jj] = __uint_as_float(r[jj]);
-        const float tot = warp_colsum16(v, lane);
-        if ((lane & 1) == 0) ctl.red[q4][c * 16 + (lane >> 1)] = tot;
-      }
-      if (lane == 0 && q4 == 0) QMLA_TRACE(101, it);
-      if (!(ok = group_sync(&ctl.grp[1], gph[1], ctl, kSiteSmLsum, p.dev_err))) break;
-      if (row < HG) {
-        const float l = (ctl.red[0][row] + ctl.red[1][row]) + (ctl.red[2][row] + ctl.red[3][row]);
-        ctl.alpha[row] = l;
-        ctl.inv[row] = 1.0f / l;  // one division per head; the rows below are multiplied
-      }
-      if (!(ok = group_sync(&ctl.grp[2], gph[2], ctl, kSiteSmL, p.dev_err))) break;
-      if (lane == 0 && q4 == 0) QMLA_TRACE(102, it);
-      if (!(ok = wwait(&ctl.pv_done, it & 1u, ctl, kSiteSmPvEpi, p.dev_err))) break;
-      tc_fence_after();
-      if (lane == 0 && q4 == 0) QMLA_TRACE(103, it);
-      const bool whole = (seg_j0 == 0) && (sc.t + 1 == sc.pu1);
-      const int h0 = ti.hg * HG;
-      const int hn = min(HG, p.heads - h0);
-      const size_t pidx = static_cast<size_t>(blockIdx.x) + sc.u;
-      // Whole segment: out = O / l (products with the per-head reciprocal);
-      // split segment: the unnormalised partial o.
-      float* const obase =
-          whole ? p.out + (static_cast<size_t>(ti.b) * p.heads + h0) * kDc : p.part_o + pidx * HG * kDc;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int P = i * 128 + row;  // position in the reconstructed row
-        float* const orow = obase + (P & ~7) + Perm<CB>::at(P & 7);
-#pragma unroll
-        for (int c = 0; c < NC; ++c) {
-          uint32_t r[16];
-          tmem_ld16(t_o + i * HG + c * 16, r);
-          float f[16];
-#pragma unroll
-          for (int v4 = 0; v4 < 4; ++v4) {
-            const float4 iv = whole ? reinterpret_cast<const float4*>(ctl.inv)[c * 4 + v4] : make_float4(1.f, 1.f, 1.f, 1.f);
-            f[4 * v4] = iv.x;
-            f[4 * v4 + 1] = iv.y;
-            f[4 * v4 + 2] = iv.z;
-            f[4 * v4 + 3] = iv.w;
-          }
-          tmem_ld_wait();
-#pragma unroll
-          for (int jj = 0; jj < 16; ++jj) {
-            const int h = c * 16 + jj;
-            if (h < hn) orow[static_cast<size_t>(h) * kDc] = __uint_as_float(r[jj]) * f[jj];
-          }
-        }
-        if (lane == 0 && q4 == 0) QMLA_TRACE(104 + i, it);
-      }
-      if (row < HG && h0 + row < p.heads) {
-        if (whole) {
-          if (p.lse != nullptr)
-            p.lse[static_cast<size_t>(ti.b) * p.heads + h0 + row] = (ctl.m_ref[row] + log2f(ctl.alpha[row])) * kLn2;
-        } else {
-          p.part_ml[(pidx * HG + row) * 2 + 0] = ctl.m_ref[row];
-          p.part_ml[(pidx * HG + row) * 2 + 1] = ctl.alpha[row];
-        }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&ctl.o_free);
-        if (q4 == 0) QMLA_TRACE(20, it);
-        if (q4 == 0) QMLA_TRACE(108, it);
-      }
-    }
-    ++it;
-  }
-  if (!ok) set_abort(ctl, p.dev_err);
 }
 
 template <int CB, int HG>
@@ -868,14 +909,15 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   if (threadIdx.x == 0) QMLA_TRACE(22, 0);
 
   if (threadIdx.x == 0) {
-    mbar_init(&ctl.tile_full, kNumDqWarps);
-    mbar_init(&ctl.s_full, 1);
-    mbar_init(&ctl.p_full, 4);
+    for (int k = 0; k < kNumChunks; ++k) mbar_init(&ctl.chunk_full[k], 4);
+    for (int j = 0; j < 3; ++j) mbar_init(&ctl.slot_free[j], 1);
     mbar_init(&ctl.pv_done, 1);
-    mbar_init(&ctl.o_free, 4);
+    mbar_init(&ctl.s_full, 1);
+    mbar_init(&ctl.p_full, kWorkers);
+    mbar_init(&ctl.o_free, kWorkers);
     mbar_init(&ctl.q_full, 1);
     mbar_init(&ctl.fin, 1);
-    for (int i = 0; i < 3; ++i) mbar_init(&ctl.grp[i], 4);
+    mbar_init(&ctl.grp, kWorkers);
     ctl.abort = 0u;
     fence_mbar_init();
   }
@@ -889,11 +931,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   const uint32_t tmem = ctl.tmem_base;
 
   Sched sc;
-  sc.init(p.prefix, p.batch * p.n_hg, blockIdx.x, gridDim.x);
-  if (warp < kNumDqWarps) {
-    dequant_role<CB, HG>(p, sc, chunks, ctl, warp, lane);
-  } else if (warp < kMmaWarp) {
-    softmax_role<CB, HG>(p, sc, chunks, ctl, tmem, warp, lane);
+  sc.init(p.prefix, p.cta_unit, p.batch * p.n_hg, blockIdx.x, gridDim.x);
+  if (warp < kWorkers) {
+    worker_role<CB, HG>(p, sc, chunks, ctl, tmem, warp, lane);
   } else {
     mma_role<HG>(p, sc, chunks, qsmem, ctl, tmem, lane);
   }
@@ -969,6 +1009,21 @@ __global__ void __launch_bounds__(kPrepThreads) prep_kernel(const Params p) {
     __syncthreads();
   }
   if (threadIdx.x == 0) p.prefix_w[p.batch * p.n_hg] = carry;
+  __syncthreads();
+  // The unit holding the first tile of every decode CTA's range (the unit u
+  // with prefix[u] <= t0 < prefix[u + 1]), so that no CTA has to search.
+  const volatile int32_t* pf = p.prefix_w;
+  const int units = p.batch * p.n_hg;
+  const int T = pf[units];
+  for (int c = threadIdx.x; c < p.grid; c += blockDim.x) {
+    const int t0 = static_cast<int>(static_cast<long long>(c) * T / p.grid);
+    int lo = 0, hi = units;
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (pf[mid] <= t0) lo = mid; else hi = mid;
+    }
+    p.cta_unit[c] = lo;
+  }
 }
 
 // First tile of CTA c's range, and the CTA whose range holds tile t.
@@ -1068,7 +1123,8 @@ DecodeWorkspace decode_workspace_layout(int batch, int heads, int grid) {
   auto up = [](size_t x) { return (x + 255) & ~static_cast<size_t>(255); };
   DecodeWorkspace w;
   w.prefix_off = 0;
-  w.part_o_off = up((units + 1) * sizeof(int32_t));
+  w.cta_off = up((units + 1) * sizeof(int32_t));
+  w.part_o_off = w.cta_off + up(static_cast<size_t>(grid) * sizeof(int32_t));
   const size_t nparts = static_cast<size_t>(grid) + units;
   w.part_ml_off = w.part_o_off + up(nparts * hg * kDc * sizeof(float));
   w.qimg_off = w.part_ml_off + up(nparts * hg * 2 * sizeof(float));
@@ -1096,6 +1152,7 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
   prm.lse = a.lse;
   prm.prefix = reinterpret_cast<const int32_t*>(ws + w.prefix_off);
   prm.prefix_w = reinterpret_cast<int32_t*>(ws + w.prefix_off);
+  prm.cta_unit = reinterpret_cast<int32_t*>(ws + w.cta_off);
   prm.part_o = reinterpret_cast<float*>(ws + w.part_o_off);
   prm.part_ml = reinterpret_cast<float*>(ws + w.part_ml_off);
   prm.qimg = ws + w.qimg_off;

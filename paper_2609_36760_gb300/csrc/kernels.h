@@ -21,7 +21,7 @@ int head_group_size(int heads);
 
 // Workspace carve-up of the decode path for `grid` CTAs.
 struct DecodeWorkspace {
-  size_t prefix_off, part_o_off, part_ml_off, qimg_off, total;
+  size_t prefix_off, cta_off, part_o_off, part_ml_off, qimg_off, total;
 };
 DecodeWorkspace decode_workspace_layout(int batch, int heads, int grid);
 
