@@ -218,7 +218,7 @@ __device__ __forceinline__ bool wwait(uint64_t* bar, uint32_t parity, Ctrl& c, u
 // cannot arrive for phase n + 2 before every warp has arrived for n + 1.
 __device__ __forceinline__ bool group_sync(Ctrl& c, uint32_t& phase, uint32_t* dev_err) {
   __syncwarp();
-  if ((threadIdx.x & 31) == 0) mbar_arrive(&c.grp);
+  mbar_arrive_if((threadIdx.x & 31) == 0 ? 1u : 0u, &c.grp);
   const bool ok = wwait(&c.grp, phase & 1u, c, kSiteGrp, dev_err);
   ++phase;
   return ok;
@@ -259,6 +259,16 @@ struct TileInfo {
   int b, hg, j, ntok;
   bool first, last;
 };
+// Segment position of the current tile, from the schedule alone (no loads).
+struct TileFlags {
+  bool first, last;
+};
+__device__ __forceinline__ TileFlags tile_flags(const Sched& s) {
+  TileFlags f;
+  f.first = (s.t == s.t0) || (s.t == s.pu0);
+  f.last = (s.t + 1 == s.t1) || (s.t + 1 == s.pu1);
+  return f;
+}
 __device__ __forceinline__ TileInfo tile_info(const Sched& s, const Params& p) {
   TileInfo ti;
   ti.b = s.u / p.n_hg;
@@ -278,20 +288,39 @@ struct Fetch {
   bool ok;
 };
 
+// Block-table entry and sequence length of one token row of a tile, loaded a
+// tile before they are needed (nothing branches on them until resolve_row).
+// The table column is clamped so that rows past the sequence end never read
+// beyond the sequence's table row.
+struct RowRef {
+  int entry, len, j;
+  bool has;
+};
+__device__ __forceinline__ RowRef row_ref(const Params& p, const Sched& s, int row) {
+  RowRef r;
+  r.has = s.valid();
+  r.entry = -1;
+  r.len = 0;
+  r.j = 0;
+  if (!r.has) return r;
+  const int b = s.u / p.n_hg;
+  r.j = s.t - s.pu0;
+  r.len = p.seq_lens[b];
+  const int lb = min(2 * r.j + (row >> 6), p.max_blocks - 1);
+  r.entry = p.table[static_cast<size_t>(b) * p.max_blocks + lb];
+  return r;
+}
 template <int CB>
-__device__ __forceinline__ const uint8_t* row_block(const Params& p, const TileInfo& ti, int row,
-                                                    bool& valid) {
-  valid = row < ti.ntok;
-  if (!valid) return nullptr;
-  const int lb = 2 * ti.j + (row >> 6);
-  const int blk = p.table[static_cast<size_t>(ti.b) * p.max_blocks + lb];
-  if (blk < 0 || blk >= p.num_blocks) {
+__device__ __forceinline__ const uint8_t* resolve_row(const Params& p, const RowRef& r, int row, bool& valid) {
+  valid = false;
+  if (!r.has || row >= min(kTileTokens, r.len - kTileTokens * r.j)) return nullptr;
+  if (r.entry < 0 || r.entry >= p.num_blocks) {
     report(p.dev_err, QMLA_DEVERR_BAD_BLOCK);
-    valid = false;
     return nullptr;
   }
+  valid = true;
   constexpr size_t kBlk = CB == 16 ? static_cast<size_t>(kBf16BlockBytes) : BlockLayout<CB == 16 ? 4 : CB>::kBytes;
-  return p.pool + static_cast<size_t>(blk) * kBlk;
+  return p.pool + static_cast<size_t>(r.entry) * kBlk;
 }
 
 template <int CB>
@@ -582,7 +611,7 @@ __device__ bool epilogue(const Params& p, const SegEnd& e, Ctrl& ctl, uint32_t t
   }
   tc_fence_before();
   __syncwarp();
-  if (lane == 0) mbar_arrive(&ctl.o_free);
+  mbar_arrive_if(lane == 0 ? 1u : 0u, &ctl.o_free);
   return true;
 }
 
@@ -613,44 +642,34 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
   Fetch f[kMyChunks];
   // BF16 cache: one chunk row (8 x 16 B) of look-ahead.
   uint4 cur[CB == 16 ? 8 : 1];
-  auto fetch_tile = [&](const Sched& s) {
-    bool valid = false;
-    const TileInfo tf = tile_info(s, p);
-    const uint8_t* blk = row_block<CB>(p, tf, row, valid);
-    if constexpr (CB != 16) {
-#pragma unroll
-      for (int kc = 0; kc < kMyChunks; ++kc) {
-        const int k = 2 * kc + par;
-        if (k < kNumChunks) f[kc] = fetch_chunk<CB>(blk, valid, k, slot);
-      }
-    }
-    return blk;
-  };
-  const uint8_t* blk_cur = nullptr;
   bool valid_cur = false;
-  if (sc.valid()) {
-    blk_cur = fetch_tile(sc);
-    valid_cur = blk_cur != nullptr;
-    if constexpr (CB == 16) {
+  const uint8_t* blk_cur = resolve_row<CB>(p, row_ref(p, sc, row), row, valid_cur);
+  if constexpr (CB != 16) {
 #pragma unroll
-      for (int i = 0; i < 8; ++i)
-        cur[i] = valid_cur ? ldg_nc_v4(blk_cur + slot * (kDqk * 2) + par * 128 + i * 16) : make_uint4(0, 0, 0, 0);
+    for (int kc = 0; kc < kMyChunks; ++kc) {
+      const int k = 2 * kc + par;
+      if (k < kNumChunks) f[kc] = fetch_chunk<CB>(blk_cur, valid_cur, k, slot);
     }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      cur[i] = valid_cur ? ldg_nc_v4(blk_cur + slot * (kDqk * 2) + par * 128 + i * 16) : make_uint4(0, 0, 0, 0);
   }
+  // Table references run one tile ahead of the block pointer they resolve to.
+  Sched nx = sc;
+  nx.next();
+  RowRef ref_nx = row_ref(p, nx, row);
 
   for (; ok && sc.valid(); sc.next()) {
-    const TileInfo ti = tile_info(sc, p);
-    if (ti.first) seg_j0 = ti.j;
-    const bool valid = row < ti.ntok;
-    Sched nx = sc;
-    nx.next();
-    const bool has_next = nx.valid();
+    const TileFlags tf = tile_flags(sc);
+    if (tf.first) seg_j0 = sc.t - sc.pu0;
+    // The next tile's block pointer (its table entry was loaded a tile ago)
+    // and the table entry of the tile after it.
     bool valid_nx = false;
-    const uint8_t* blk_nx = nullptr;
-    if (has_next) {
-      const TileInfo tn = tile_info(nx, p);
-      blk_nx = row_block<CB>(p, tn, row, valid_nx);
-    }
+    const uint8_t* blk_nx = resolve_row<CB>(p, ref_nx, row, valid_nx);
+    Sched nn = nx;
+    nn.next();
+    const RowRef ref_nn = row_ref(p, nn, row);
     if (lane == 0 && warp == 0) QMLA_TRACE(0, it);
 
     // ---- dequantise this tile, chunk by chunk as the previous PV frees the slots
@@ -659,6 +678,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       const int k = 2 * kc + par;
       if (k >= kNumChunks) break;
       if (!(ok = wwait(slot_bar(ctl, k), (it & 1u) ^ 1u, ctl, kSiteDqSlot, p.dev_err))) break;
+      if (lane == 0) QMLA_TRACE(88 + warp, it);  // (overwritten per chunk: last slot wait)
       if constexpr (CB == 16) {
         uint4 nxt[8];
         const int kn = k + 2;
@@ -680,12 +700,17 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       }
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl.chunk_full[k]);
+      mbar_arrive_if(lane == 0 ? 1u : 0u, &ctl.chunk_full[k]);
+      if (lane == 0) QMLA_TRACE(48 + warp * 5 + kc, it);
     }
     if (!ok) break;
     if (lane == 0) QMLA_TRACE(32 + warp, it);
     blk_cur = blk_nx;
     valid_cur = valid_nx;
+    nx = nn;
+    ref_nx = ref_nn;
+    const TileInfo ti = tile_info(sc, p);  // ntok of this tile for the softmax (loaded long ago)
+    const bool valid = row < ti.ntok;
 
     // ---- the previous segment's results (its last PV completed: chunks 6..8 were waited for)
     if (pending) {
@@ -773,10 +798,8 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     fence_proxy_async_smem();
     tc_fence_before();
     __syncwarp();
-    if (lane == 0) {
-      mbar_arrive(&ctl.p_full);
-      if (warp == 0) QMLA_TRACE(19, it);
-    }
+    mbar_arrive_if(lane == 0 ? 1u : 0u, &ctl.p_full);
+    if (lane == 0 && warp == 0) QMLA_TRACE(19, it);
     if (ti.last) {
       pending = true;
       pend.b = ti.b;
@@ -808,16 +831,22 @@ __device__ __forceinline__ void issue_query(const Params& p, int unit, uint8_t* 
   for (int k = 0; k < kNumChunks; ++k) bulk_g2s(qsmem + k * HG * 128, src + k * HG * 128, HG * 128, &ctl.q_full);
 }
 
-// The MMA warp walks the schedule and waits on every lane; one elected lane
-// issues the MMAs, the commits (a commit tracks the MMAs issued by the
-// committing thread) and the query copies. QK starts on each chunk as soon
-// as it is written; PV commits after each 128-channel block so that the next
-// tile's dequantisation can refill those slots. Descriptors are advanced by
-// adding (byte offset >> 4) to their start-address field.
+// Bounded wait of the single MMA thread (no warp-collective operations: the
+// other lanes of its warp have exited).
+__device__ __forceinline__ bool twait(uint64_t* bar, uint32_t parity, Ctrl& c, uint32_t site, uint32_t* dev_err) {
+  return wait_ok(mbar_wait(bar, parity, kWaitNs, &c.abort), site, c, dev_err);
+}
+
+// One thread issues every MMA, commit and query copy (the other lanes of its
+// warp exit at the start: a warp whose lane 0 issues or waits while the other
+// lanes sit at a re-convergence point was measured to issue MMAs and wake up
+// far more slowly on sm_103a). A commit tracks the MMAs issued by the
+// committing thread. QK starts on each chunk as soon as it is written; PV
+// commits after each 128-channel block so that the next tile's
+// dequantisation can refill those slots. Descriptors are advanced by adding
+// (byte offset >> 4) to their start-address field.
 template <int HG>
-__device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint8_t* qsmem, Ctrl& ctl,
-                         uint32_t tmem, int lane) {
-  const bool leader = lane == 0;
+__device__ void mma_thread(const Params& p, Sched sc, uint32_t chunks, uint8_t* qsmem, Ctrl& ctl, uint32_t tmem) {
   constexpr uint32_t kIdQK = idesc_f16_f32(128, HG, false, false);
   constexpr uint32_t kIdPV = idesc_f16_f32(128, HG, true, true);
   constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
@@ -831,70 +860,54 @@ __device__ void mma_role(const Params& p, Sched sc, uint32_t chunks, uint8_t* qs
   const uint64_t pv_b0 = smem_desc(ptile, 16 * kSboP, kSboP, swz_mode_for_row(kRB));
   uint32_t it = 0, seg = 0;
   bool ok = true;
-  if (sc.valid() && leader) issue_query<HG>(p, sc.u, qsmem, ctl);
+  if (sc.valid()) issue_query<HG>(p, sc.u, qsmem, ctl);
   for (; ok && sc.valid(); sc.next()) {
-    const TileInfo ti = tile_info(sc, p);
-    if (ti.first && !(ok = wwait(&ctl.q_full, seg & 1u, ctl, kSiteMmaQFull, p.dev_err))) break;
+    const TileFlags ti = tile_flags(sc);
+    if (ti.first && !(ok = twait(&ctl.q_full, seg & 1u, ctl, kSiteMmaQFull, p.dev_err))) break;
     // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576), chunk by chunk.
-#pragma unroll 1
-    for (int k = 0; k < kNumChunks; ++k) {
-      if (!(ok = wwait(&ctl.chunk_full[k], it & 1u, ctl, kSiteMmaChunk, p.dev_err))) break;
-      tc_fence_after();
-      if (leader) {
-        if (k == 0) QMLA_TRACE(11, it);
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
-          const uint64_t ad = qk_a0 + static_cast<uint64_t>((k * kChunkBytes + kk * 32) >> 4);
-          const uint64_t bd = qk_b0 + static_cast<uint64_t>((k * HG * 128 + kk * 32) >> 4);
-          umma_f16_ss(t_s, ad, bd, kIdQK, (k | kk) != 0 ? 1u : 0u);
-        }
-      }
-      __syncwarp();
+    for (int k = 0; k < kNumChunks; ++k) {
+      if (!(ok = twait(&ctl.chunk_full[k], it & 1u, ctl, kSiteMmaChunk, p.dev_err))) break;
+      tc_fence_after();
+      QMLA_TRACE(112 + k, it);
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)
+        umma_f16_ss(t_s, qk_a0 + static_cast<uint64_t>((k * kChunkBytes + kk * 32) >> 4),
+                    qk_b0 + static_cast<uint64_t>((k * HG * 128 + kk * 32) >> 4), kIdQK, (k | kk) != 0 ? 1u : 0u);
     }
     if (!ok) break;
-    if (leader) {
-      umma_commit(&ctl.s_full);
-      QMLA_TRACE(12, it);
-    }
-    __syncwarp();
-    if (!(ok = wwait(&ctl.p_full, it & 1u, ctl, kSiteMmaPFull, p.dev_err))) break;
-    if (leader) QMLA_TRACE(14, it);
-    if (ti.last && leader) {
+    umma_commit(&ctl.s_full);
+    QMLA_TRACE(12, it);
+    if (!(ok = twait(&ctl.p_full, it & 1u, ctl, kSiteMmaPFull, p.dev_err))) break;
+    QMLA_TRACE(14, it);
+    if (ti.last) {
       // The softmax only signals P after this tile's QK has completed, so the
       // query tile is free: start copying the next segment's query now.
       Sched nx = sc;
       nx.next();
       if (nx.valid()) issue_query<HG>(p, nx.u, qsmem, ctl);
     }
-    if (ti.first && seg > 0 &&
-        !(ok = wwait(&ctl.o_free, (seg - 1) & 1u, ctl, kSiteMmaOFree, p.dev_err)))
-      break;
+    if (ti.first && seg > 0 && !(ok = twait(&ctl.o_free, (seg - 1) & 1u, ctl, kSiteMmaOFree, p.dev_err))) break;
     tc_fence_after();
-    if (leader) {
-      // O^T[c, h] += sum_t C_hat[t, c] P^T[t, h], 4 x 128 channels, K = 128 tokens.
+    // O^T[c, h] += sum_t C_hat[t, c] P^T[t, h], 4 x 128 channels, K = 128 tokens.
+    const uint32_t acc0 = ti.first ? 0u : 1u;
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < 4; ++i) {
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-          const uint64_t ad = pv_a0 + static_cast<uint64_t>((2 * i * kChunkBytes + kk * 2048) >> 4);
-          const uint64_t bd = pv_b0 + static_cast<uint64_t>((kk * 2 * kSboP) >> 4);
-          umma_f16_ss(tmem + i * HG, ad, bd, kIdPV, (ti.first && kk == 0) ? 0u : 1u);
-        }
-        umma_commit(i < 3 ? &ctl.slot_free[i] : &ctl.pv_done);
-      }
-      QMLA_TRACE(15, it);
+      for (int kk = 0; kk < 8; ++kk)
+        umma_f16_ss(tmem + i * HG, pv_a0 + static_cast<uint64_t>((2 * i * kChunkBytes + kk * 2048) >> 4),
+                    pv_b0 + static_cast<uint64_t>((kk * 2 * kSboP) >> 4), kIdPV, kk == 0 ? acc0 : 1u);
+      umma_commit(i < 3 ? &ctl.slot_free[i] : &ctl.pv_done);
     }
-    __syncwarp();
+    QMLA_TRACE(15, it);
     ++it;
     if (ti.last) ++seg;
   }
-  if (!ok && leader) set_abort(ctl, p.dev_err);
+  if (!ok) set_abort(ctl, p.dev_err);
   // Every MMA and copy must have landed before TMEM and shared memory are
   // released; this wait ignores the abort flag.
-  if (leader) umma_commit(&ctl.fin);
-  __syncwarp();
+  umma_commit(&ctl.fin);
   wait_ok(mbar_wait(&ctl.fin, 0, kWaitNs, nullptr), kSiteMmaFin, ctl, p.dev_err);
-  __syncwarp();
 }
 
 template <int CB, int HG>
@@ -921,7 +934,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
     ctl.abort = 0u;
     fence_mbar_init();
   }
-  if (warp == kMmaWarp) {
+  if (warp == 0) {  // worker warp 0 owns the TMEM allocation
     tmem_alloc(&ctl.tmem_base, Cfg<HG>::kTmemCols);
     tmem_relinquish();
   }
@@ -929,17 +942,18 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = ctl.tmem_base;
+  if (warp == kMmaWarp && lane != 0) return;  // the MMA role is a single thread
 
   Sched sc;
   sc.init(p.prefix, p.cta_unit, p.batch * p.n_hg, blockIdx.x, gridDim.x);
   if (warp < kWorkers) {
     worker_role<CB, HG>(p, sc, chunks, ctl, tmem, warp, lane);
   } else {
-    mma_role<HG>(p, sc, chunks, qsmem, ctl, tmem, lane);
+    mma_thread<HG>(p, sc, chunks, qsmem, ctl, tmem);
   }
   tc_fence_before();
-  __syncthreads();
-  if (warp == kMmaWarp) {
+  __syncthreads();  // the exited lanes of the MMA warp do not take part
+  if (warp == 0) {
     tc_fence_after();
     tmem_dealloc(tmem, Cfg<HG>::kTmemCols);
   }
