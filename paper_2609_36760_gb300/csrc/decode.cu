@@ -65,9 +65,19 @@ constexpr int kTraceCtas = 8, kTraceEvents = 128, kTraceTiles = 32;
       p.trace[(static_cast<size_t>(blockIdx.x) * kTraceEvents + (ev)) * kTraceTiles + (tile)] = \
           clock64();                                                                             \
   } while (0)
+// All CTAs: wall-clock start/end (%globaltimer), SM id and tile count after the event area.
+#define QMLA_TRACE_CTA(slot, value)                                                                       \
+  do {                                                                                                    \
+    if (p.trace != nullptr)                                                                               \
+      p.trace[static_cast<size_t>(kTraceCtas) * kTraceEvents * kTraceTiles + blockIdx.x * 4 + (slot)] = \
+          (value);                                                                                        \
+  } while (0)
 #else
 #define QMLA_TRACE(ev, tile) \
   do {                       \
+  } while (0)
+#define QMLA_TRACE_CTA(slot, value) \
+  do {                              \
   } while (0)
 #endif
 
@@ -101,11 +111,13 @@ struct __align__(16) Ctrl {
   // slot) are free and O^T holds the sum through that tile.
   uint64_t chunk_full[kNumChunks];
   uint64_t slot_free[3];
-  uint64_t pv_done, s_full, p_full, o_free, q_full, fin;
+  // p_full: every worker wrote its part of P (one arrive per warp). p_fixed: after a
+  // rescale, P was rewritten against the raised reference.
+  uint64_t pv_done, s_full, p_full, p_fixed, o_free, q_full, fin;
   uint64_t grp;  // barrier among the worker warps (one arrive per warp, reused in sequence)
   uint32_t tmem_base;
   uint32_t abort;
-  uint32_t vote[2][kWorkers];
+  uint32_t resc_tile;  // it + 1 when tile it needs a rescale (written before p_full)
   alignas(16) float m_ref[64];  // read as float4
   alignas(16) float alpha[64];
   alignas(16) float inv[64];  // 1 / l per head at a segment end, read as float4
@@ -632,7 +644,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
   const uint32_t ptile = chunks + 8 * kChunkBytes;
   const float sl2 = p.scale_log2;
   constexpr int kMyChunks = 5;  // chunks per parity, rounded up (parity 1 has 4)
-  uint32_t it = 0, gph = 0;
+  uint32_t it = 0, gph = 0, nresc = 0;
   int seg_j0 = 0;
   bool ok = true;
   bool pending = false;  // the previous tile ended a segment whose epilogue is still due
@@ -736,18 +748,23 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     }
     uint32_t pk[C::kPerWarp / 2];
     const bool over = compute_p<HG>(t_s, ctl.m_ref + cb0, sl2, valid, ptile, row, piece0, pk);
-    uint32_t* vote = ctl.vote[it & 1u];
-    const uint32_t any = __any_sync(0xffffffffu, over);
-    if (lane == 0) vote[warp] = any;
-    if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
+    // A weight above 2^8 anywhere in the tile asks for a rescale; the flag is
+    // written before p_full, so whoever has seen p_full complete reads it.
+    if (__any_sync(0xffffffffu, over) && lane == 0) *reinterpret_cast<volatile uint32_t*>(&ctl.resc_tile) = it + 1;
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncwarp();
+    mbar_arrive_if(lane == 0 ? 1u : 0u, &ctl.p_full);
+    if (lane == 0 && warp == 0) QMLA_TRACE(19, it);
+    // Off the MMA thread's path from here: learn whether any warp asked for a rescale.
+    if (!(ok = wwait(&ctl.p_full, it & 1u, ctl, kSiteGrp, p.dev_err))) break;
     if (lane == 0 && warp == 0) QMLA_TRACE(17, it);
-    uint32_t anyv = 0;
-#pragma unroll
-    for (int w = 0; w < kWorkers; ++w) anyv |= vote[w];
-    if (anyv != 0u) {
+    if (*reinterpret_cast<volatile uint32_t*>(&ctl.resc_tile) == it + 1) {
       // Raise the reference to the running max; O and the row sums were
       // accumulated against the old one and are scaled by alpha = 2^(m_old - m_new).
-      // The previous PV has completed (its slots were waited for above).
+      // The previous PV has completed (its slots were waited for above); the
+      // MMA thread waits on p_fixed before this tile's PV.
+      tc_fence_after();
       warp_tile_max<HG>(t_s, sl2, valid, &ctl.red[q4][cb0], lane);
       if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
       if (threadIdx.x < HG) {
@@ -777,8 +794,13 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
         tmem_st_wait();
       }
       compute_p<HG>(t_s, ctl.m_ref + cb0, sl2, valid, ptile, row, piece0, pk);
+      fence_proxy_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      mbar_arrive_if(lane == 0 ? 1u : 0u, &ctl.p_fixed);
+      ++nresc;
     }
-    // Row sums of the fp16 weights the PV MMA multiplies with.
+    // Row sums of the fp16 weights the PV MMA multiplies with (no MMA reads them).
 #pragma unroll
     for (int c = 0; c < C::kN; ++c) {
       uint32_t r[C::kW];
@@ -795,11 +817,6 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       tmem_st(t_l + c * C::kW, r);
     }
     tmem_st_wait();
-    fence_proxy_async_smem();
-    tc_fence_before();
-    __syncwarp();
-    mbar_arrive_if(lane == 0 ? 1u : 0u, &ctl.p_full);
-    if (lane == 0 && warp == 0) QMLA_TRACE(19, it);
     if (ti.last) {
       pending = true;
       pend.b = ti.b;
@@ -858,18 +875,23 @@ __device__ void mma_thread(const Params& p, Sched sc, uint32_t chunks, uint8_t* 
   const uint64_t qk_b0 = smem_desc(qbase, 16, 1024, SWZ_128B);
   const uint64_t pv_a0 = smem_desc(chunks, kChunkBytes, 1024, SWZ_128B);
   const uint64_t pv_b0 = smem_desc(ptile, 16 * kSboP, kSboP, swz_mode_for_row(kRB));
-  uint32_t it = 0, seg = 0;
+  uint32_t it = 0, seg = 0, nresc = 0;
   bool ok = true;
   if (sc.valid()) issue_query<HG>(p, sc.u, qsmem, ctl);
   for (; ok && sc.valid(); sc.next()) {
     const TileFlags ti = tile_flags(sc);
     if (ti.first && !(ok = twait(&ctl.q_full, seg & 1u, ctl, kSiteMmaQFull, p.dev_err))) break;
-    // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576), chunk by chunk.
+    // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576), chunk by
+    // chunk. The next chunk's barrier is probed before this chunk's MMAs are
+    // issued, so the probe's latency overlaps them; only a chunk that was not
+    // yet written takes the (bounded) wait.
+    bool ready = mbar_test(&ctl.chunk_full[0], it & 1u);
 #pragma unroll
     for (int k = 0; k < kNumChunks; ++k) {
-      if (!(ok = twait(&ctl.chunk_full[k], it & 1u, ctl, kSiteMmaChunk, p.dev_err))) break;
+      if (!ready && !(ok = twait(&ctl.chunk_full[k], it & 1u, ctl, kSiteMmaChunk, p.dev_err))) break;
       tc_fence_after();
       QMLA_TRACE(112 + k, it);
+      if (k + 1 < kNumChunks) ready = mbar_test(&ctl.chunk_full[k + 1], it & 1u);
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk)
         umma_f16_ss(t_s, qk_a0 + static_cast<uint64_t>((k * kChunkBytes + kk * 32) >> 4),
@@ -879,6 +901,10 @@ __device__ void mma_thread(const Params& p, Sched sc, uint32_t chunks, uint8_t* 
     umma_commit(&ctl.s_full);
     QMLA_TRACE(12, it);
     if (!(ok = twait(&ctl.p_full, it & 1u, ctl, kSiteMmaPFull, p.dev_err))) break;
+    if (*reinterpret_cast<volatile uint32_t*>(&ctl.resc_tile) == it + 1) {
+      if (!(ok = twait(&ctl.p_fixed, nresc & 1u, ctl, kSiteMmaPFull, p.dev_err))) break;
+      ++nresc;
+    }
     QMLA_TRACE(14, it);
     if (ti.last) {
       // The softmax only signals P after this tile's QK has completed, so the
@@ -919,7 +945,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   Ctrl& ctl = *reinterpret_cast<Ctrl*>(smem + kNumChunks * kChunkBytes + Cfg<HG>::kQBytes);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  if (threadIdx.x == 0) QMLA_TRACE(22, 0);
+  if (threadIdx.x == 0) {
+    QMLA_TRACE(22, 0);
+    QMLA_TRACE_CTA(0, globaltimer_ns());
+    uint32_t smid;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(smid));
+    QMLA_TRACE_CTA(2, smid);
+  }
 
   if (threadIdx.x == 0) {
     for (int k = 0; k < kNumChunks; ++k) mbar_init(&ctl.chunk_full[k], 4);
@@ -927,6 +959,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
     mbar_init(&ctl.pv_done, 1);
     mbar_init(&ctl.s_full, 1);
     mbar_init(&ctl.p_full, kWorkers);
+    mbar_init(&ctl.p_fixed, kWorkers);
+    ctl.resc_tile = 0u;
     mbar_init(&ctl.o_free, kWorkers);
     mbar_init(&ctl.q_full, 1);
     mbar_init(&ctl.fin, 1);
@@ -957,7 +991,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
     tc_fence_after();
     tmem_dealloc(tmem, Cfg<HG>::kTmemCols);
   }
-  if (threadIdx.x == 0) QMLA_TRACE(23, 0);
+  if (threadIdx.x == 0) {
+    QMLA_TRACE(23, 0);
+    QMLA_TRACE_CTA(1, globaltimer_ns());
+    QMLA_TRACE_CTA(3, static_cast<unsigned long long>(sc.t1 - sc.t0));
+  }
 }
 
 // ------------------------------------------------------------ prep / combine
