@@ -95,7 +95,11 @@ struct Params {
   float* lse;
   const int32_t* prefix;
   int32_t* prefix_w;
-  int32_t* cta_unit;  // [grid]: unit holding each CTA's first tile (written with the prefix)
+  // [grid] per CTA, written by the prep kernel with the prefix: {unit of the first
+  // tile, prefix[unit], prefix[unit + 1], total tiles} and, for the first tile,
+  // {table entry of rows 0..63, of rows 64..127, sequence length, tile index}.
+  int4* cta_info;
+  int4* cta_first;
   float* part_o;   // [(grid + units)][HG][512]
   float* part_ml;  // [(grid + units)][HG][2]
   uint8_t* qimg;   // [units][9][HG][128 B]: swizzled fp16 query tiles
@@ -241,20 +245,18 @@ struct Sched {
   const int32_t* prefix;
   int t0, t1, t, u, pu0, pu1;
   int units;
-  // cu[cta] is the unit holding tile t0 (found once by the prep kernel).
-  __device__ void init(const int32_t* pf, const int32_t* cu, int units_, int cta, int grid) {
+  // info = {unit holding tile t0, prefix[unit], prefix[unit + 1], total tiles}
+  // for this CTA (found once by the prep kernel).
+  __device__ void init(const int32_t* pf, int4 info, int units_, int cta, int grid) {
     prefix = pf;
     units = units_;
-    const int T = pf[units];
+    const int T = info.w;
     t0 = static_cast<int>(static_cast<long long>(cta) * T / grid);
     t1 = static_cast<int>(static_cast<long long>(cta + 1) * T / grid);
     t = t0;
-    u = 0;
-    pu0 = pu1 = 0;
-    if (t0 >= t1) return;
-    u = cu[cta];
-    pu0 = pf[u];
-    pu1 = pf[u + 1];
+    u = info.x;
+    pu0 = info.y;
+    pu1 = info.z;
   }
   __device__ bool valid() const { return t < t1; }
   __device__ void next() {
@@ -655,7 +657,15 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
   // BF16 cache: one chunk row (8 x 16 B) of look-ahead.
   uint4 cur[CB == 16 ? 8 : 1];
   bool valid_cur = false;
-  const uint8_t* blk_cur = resolve_row<CB>(p, row_ref(p, sc, row), row, valid_cur);
+  RowRef ref0;  // the first tile's reference, prepared by the prep kernel
+  {
+    const int4 fr = p.cta_first[blockIdx.x];
+    ref0.has = sc.valid();
+    ref0.entry = row < 64 ? fr.x : fr.y;
+    ref0.len = fr.z;
+    ref0.j = fr.w;
+  }
+  const uint8_t* blk_cur = resolve_row<CB>(p, ref0, row, valid_cur);
   if constexpr (CB != 16) {
 #pragma unroll
     for (int kc = 0; kc < kMyChunks; ++kc) {
@@ -885,8 +895,10 @@ __device__ void mma_thread(const Params& p, Sched sc, uint32_t chunks, uint8_t* 
     // chunk. The next chunk's barrier is probed before this chunk's MMAs are
     // issued, so the probe's latency overlaps them; only a chunk that was not
     // yet written takes the (bounded) wait.
+    // (Unrolled by three: fully unrolled, the first tile after a cold start
+    // spends thousands of cycles fetching the loop's instructions.)
     bool ready = mbar_test(&ctl.chunk_full[0], it & 1u);
-#pragma unroll
+#pragma unroll 3
     for (int k = 0; k < kNumChunks; ++k) {
       if (!ready && !(ok = twait(&ctl.chunk_full[k], it & 1u, ctl, kSiteMmaChunk, p.dev_err))) break;
       tc_fence_after();
@@ -979,7 +991,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   if (warp == kMmaWarp && lane != 0) return;  // the MMA role is a single thread
 
   Sched sc;
-  sc.init(p.prefix, p.cta_unit, p.batch * p.n_hg, blockIdx.x, gridDim.x);
+  sc.init(p.prefix, p.cta_info[blockIdx.x], p.batch * p.n_hg, blockIdx.x, gridDim.x);
   if (warp < kWorkers) {
     worker_role<CB, HG>(p, sc, chunks, ctl, tmem, warp, lane);
   } else {
@@ -1074,7 +1086,16 @@ __global__ void __launch_bounds__(kPrepThreads) prep_kernel(const Params p) {
       const int mid = (lo + hi) >> 1;
       if (pf[mid] <= t0) lo = mid; else hi = mid;
     }
-    p.cta_unit[c] = lo;
+    const int pu0 = pf[lo], pu1 = pf[lo + 1];
+    p.cta_info[c] = make_int4(lo, pu0, pu1, T);
+    // The first tile's block-table entries (clamped column, like row_ref) and length.
+    const int b = lo / p.n_hg;
+    const int j = t0 - pu0;
+    const int32_t* trow = p.table + static_cast<size_t>(b) * p.max_blocks;
+    const bool any = t0 < static_cast<int>(static_cast<long long>(c + 1) * T / p.grid);
+    p.cta_first[c] = any ? make_int4(trow[min(2 * j, p.max_blocks - 1)], trow[min(2 * j + 1, p.max_blocks - 1)],
+                                     p.seq_lens[b], j)
+                         : make_int4(-1, -1, 0, 0);
   }
 }
 
@@ -1176,7 +1197,7 @@ DecodeWorkspace decode_workspace_layout(int batch, int heads, int grid) {
   DecodeWorkspace w;
   w.prefix_off = 0;
   w.cta_off = up((units + 1) * sizeof(int32_t));
-  w.part_o_off = w.cta_off + up(static_cast<size_t>(grid) * sizeof(int32_t));
+  w.part_o_off = w.cta_off + up(static_cast<size_t>(grid) * 2 * sizeof(int4));
   const size_t nparts = static_cast<size_t>(grid) + units;
   w.part_ml_off = w.part_o_off + up(nparts * hg * kDc * sizeof(float));
   w.qimg_off = w.part_ml_off + up(nparts * hg * 2 * sizeof(float));
@@ -1204,7 +1225,8 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
   prm.lse = a.lse;
   prm.prefix = reinterpret_cast<const int32_t*>(ws + w.prefix_off);
   prm.prefix_w = reinterpret_cast<int32_t*>(ws + w.prefix_off);
-  prm.cta_unit = reinterpret_cast<int32_t*>(ws + w.cta_off);
+  prm.cta_info = reinterpret_cast<int4*>(ws + w.cta_off);
+  prm.cta_first = prm.cta_info + a.grid;
   prm.part_o = reinterpret_cast<float*>(ws + w.part_o_off);
   prm.part_ml = reinterpret_cast<float*>(ws + w.part_ml_off);
   prm.qimg = ws + w.qimg_off;
