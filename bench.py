@@ -139,8 +139,15 @@ def profile_traffic(kernel_file_hash: str):
 
 
 def decode_cu_hash() -> str:
-    with open(os.path.join(ROOT, "paper_2609_36760_gb300", "csrc", "decode.cu"), "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()
+    """sha256 over every CUDA source and header of the library (sorted by name),
+    so a traffic figure taken on another version of the kernel is not used."""
+    d = os.path.join(ROOT, "paper_2609_36760_gb300", "csrc")
+    h = hashlib.sha256()
+    for name in sorted(os.listdir(d)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(d, name), "rb") as f:
+                h.update(name.encode() + b"\0" + f.read())
+    return h.hexdigest()
 
 
 # ------------------------------------------------------------------ native
