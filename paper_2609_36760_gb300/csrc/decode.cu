@@ -100,6 +100,7 @@ struct Params {
   // {table entry of rows 0..63, of rows 64..127, sequence length, tile index}.
   int4* cta_info;
   int4* cta_first;
+  int32_t* cta_t0;  // [grid + 1]: first tile of each CTA's range (cta_t0[grid] = total tiles)
   float* part_o;   // [(grid + units)][HG][512]
   float* part_ml;  // [(grid + units)][HG][2]
   uint8_t* qimg;   // [units][9][HG][128 B]: swizzled fp16 query tiles
@@ -1096,59 +1097,69 @@ __global__ void __launch_bounds__(kPrepThreads) prep_kernel(const Params p) {
     p.cta_first[c] = any ? make_int4(trow[min(2 * j, p.max_blocks - 1)], trow[min(2 * j + 1, p.max_blocks - 1)],
                                      p.seq_lens[b], j)
                          : make_int4(-1, -1, 0, 0);
+    p.cta_t0[c] = t0;
   }
+  if (threadIdx.x == 0) p.cta_t0[p.grid] = T;
 }
 
-// First tile of CTA c's range, and the CTA whose range holds tile t.
-__device__ __forceinline__ int cta_start(int c, int T, int grid) {
-  return static_cast<int>(static_cast<long long>(c) * T / grid);
-}
+// The CTA whose range holds tile t (CTA c's range starts at c * T / grid).
 __device__ __forceinline__ int cta_of(int t, int T, int grid) {
   return static_cast<int>((static_cast<long long>(t + 1) * grid - 1) / T);
 }
 
-// One block per (unit, head): merges that head's partials with the App. C.5
-// rule; each thread owns 4 of the 512 channels.
+// Merges the partials of split units with the App. C.5 rule, as a running
+// merge: M = max m_j, l = sum 2^(m_j - M) l_j, O = sum 2^(m_j - M) o_j / l (the
+// running form rescales by 2^(M_old - M_new) when M grows). One block per
+// (unit, 4 heads), a warp per head, 16 channels per thread; the loads of the
+// next partial do not depend on the previous one's arithmetic.
 template <int HG>
 __global__ void __launch_bounds__(128) combine_kernel(const Params p) {
   const int u = blockIdx.x;
-  const int h = blockIdx.y;
+  const int h = blockIdx.y * 4 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
   const int units = p.batch * p.n_hg;
   const int b = u / p.n_hg;
   const int h0 = (u - b * p.n_hg) * HG;
-  if (h0 + h >= p.heads) return;
+  if (h >= HG || h0 + h >= p.heads) return;
   const int P0 = p.prefix[u], P1 = p.prefix[u + 1], T = p.prefix[units];
-  float4* out = reinterpret_cast<float4*>(p.out + (static_cast<size_t>(b) * p.heads + h0 + h) * kDc);
-  const int q = threadIdx.x;
+  float4* out = reinterpret_cast<float4*>(p.out + (static_cast<size_t>(b) * p.heads + h0 + h) * kDc) + lane * 4;
   if (P0 == P1) {
-    out[q] = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (p.lse != nullptr && q == 0) p.lse[static_cast<size_t>(b) * p.heads + h0 + h] = -INFINITY;
+#pragma unroll
+    for (int v = 0; v < 4; ++v) out[v] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (p.lse != nullptr && lane == 0) p.lse[static_cast<size_t>(b) * p.heads + h0 + h] = -INFINITY;
     return;
   }
   const int c0 = cta_of(P0, T, p.grid), c1 = cta_of(P1 - 1, T, p.grid);
   if (c0 == c1) return;  // one CTA covered the whole unit and wrote the result
-  // CTAs between c0 and c1 with an empty range wrote no partial.
-  float M = -INFINITY;
+  float M = -INFINITY, l = 0.0f;
+  float4 acc[4];
+#pragma unroll
+  for (int v = 0; v < 4; ++v) acc[v] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 2
   for (int c = c0; c <= c1; ++c) {
-    if (cta_start(c, T, p.grid) == cta_start(c + 1, T, p.grid)) continue;
-    M = fmaxf(M, p.part_ml[((static_cast<size_t>(c) + u) * HG + h) * 2]);
-  }
-  float s = 0.0f;
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int c = c0; c <= c1; ++c) {
-    if (cta_start(c, T, p.grid) == cta_start(c + 1, T, p.grid)) continue;
+    if (p.cta_t0[c] == p.cta_t0[c + 1]) continue;  // an empty range wrote no partial
     const size_t pi = (static_cast<size_t>(c) + u) * HG + h;
-    const float w = exp2f(p.part_ml[pi * 2] - M);
-    s += w * p.part_ml[pi * 2 + 1];
-    const float4 o = reinterpret_cast<const float4*>(p.part_o + pi * kDc)[q];
-    acc.x += w * o.x;
-    acc.y += w * o.y;
-    acc.z += w * o.z;
-    acc.w += w * o.w;
+    const float2 ml = *reinterpret_cast<const float2*>(p.part_ml + pi * 2);
+    const float4* o = reinterpret_cast<const float4*>(p.part_o + pi * kDc) + lane * 4;
+    float4 ov[4];
+#pragma unroll
+    for (int v = 0; v < 4; ++v) ov[v] = o[v];
+    const float Mn = fmaxf(M, ml.x);
+    const float a = exp2f(M - Mn), w = exp2f(ml.x - Mn);
+    l = l * a + w * ml.y;
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+      acc[v].x = acc[v].x * a + w * ov[v].x;
+      acc[v].y = acc[v].y * a + w * ov[v].y;
+      acc[v].z = acc[v].z * a + w * ov[v].z;
+      acc[v].w = acc[v].w * a + w * ov[v].w;
+    }
+    M = Mn;
   }
-  const float inv = 1.0f / s;
-  out[q] = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
-  if (q == 0 && p.lse != nullptr) p.lse[static_cast<size_t>(b) * p.heads + h0 + h] = (M + log2f(s)) * kLn2;
+  const float inv = 1.0f / l;
+#pragma unroll
+  for (int v = 0; v < 4; ++v) out[v] = make_float4(acc[v].x * inv, acc[v].y * inv, acc[v].z * inv, acc[v].w * inv);
+  if (lane == 0 && p.lse != nullptr) p.lse[static_cast<size_t>(b) * p.heads + h0 + h] = (M + log2f(l)) * kLn2;
 }
 
 template <int CB, int HG>
@@ -1171,7 +1182,7 @@ cudaError_t launch_impl(const Params& prm, cudaStream_t stream, cudaEvent_t ev0,
   decode_main<CB, HG><<<prm.grid, kThreads, Cfg<HG>::kSmem, stream>>>(prm);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (ev1 != nullptr && (e = cudaEventRecord(ev1, stream)) != cudaSuccess) return e;
-  combine_kernel<HG><<<dim3(static_cast<unsigned>(units), HG), 128, 0, stream>>>(prm);
+  combine_kernel<HG><<<dim3(static_cast<unsigned>(units), (HG + 3) / 4), 128, 0, stream>>>(prm);
   return cudaGetLastError();
 }
 
@@ -1197,7 +1208,7 @@ DecodeWorkspace decode_workspace_layout(int batch, int heads, int grid) {
   DecodeWorkspace w;
   w.prefix_off = 0;
   w.cta_off = up((units + 1) * sizeof(int32_t));
-  w.part_o_off = w.cta_off + up(static_cast<size_t>(grid) * 2 * sizeof(int4));
+  w.part_o_off = w.cta_off + up(static_cast<size_t>(grid) * 2 * sizeof(int4) + (grid + 1) * sizeof(int32_t));
   const size_t nparts = static_cast<size_t>(grid) + units;
   w.part_ml_off = w.part_o_off + up(nparts * hg * kDc * sizeof(float));
   w.qimg_off = w.part_ml_off + up(nparts * hg * 2 * sizeof(float));
@@ -1227,6 +1238,7 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
   prm.prefix_w = reinterpret_cast<int32_t*>(ws + w.prefix_off);
   prm.cta_info = reinterpret_cast<int4*>(ws + w.cta_off);
   prm.cta_first = prm.cta_info + a.grid;
+  prm.cta_t0 = reinterpret_cast<int32_t*>(prm.cta_first + a.grid);
   prm.part_o = reinterpret_cast<float*>(ws + w.part_o_off);
   prm.part_ml = reinterpret_cast<float*>(ws + w.part_ml_off);
   prm.qimg = ws + w.qimg_off;
