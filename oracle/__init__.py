@@ -13,8 +13,11 @@ layout     this library's 64-token block byte layout, writer and reader
 attention  dequantisation, absorbed MLA decode attention in fp64 (Eq. mla_compact)
            and the split-result merge (App. C.5, global attention normalisation)
 storage    the persistent-storage closed form (App. C.5, Eq. physical_cache_storage)
+protection sink4/local128 BF16 protection: the protected set, this library's
+           protection-buffer rows and writer rule, protected attention (App. C.5,
+           "BF16 protection and cache lifecycle")
 
 Every function is pinned by tests under ``tests/test_oracle_*.py``; nothing in
 this package is marked "parity unpinned".
 """
-from . import attention, layout, quantizer, storage  # noqa: F401
+from . import attention, layout, protection, quantizer, storage  # noqa: F401
