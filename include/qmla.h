@@ -117,6 +117,37 @@ int qmla_bf16_append(void* pool_dev, int num_blocks, const uint16_t* latent_dev,
                      const int32_t* positions_dev, int n, const int32_t* block_table_dev,
                      int num_seqs, int max_blocks, uint32_t* dev_err_dev, qmla_stream_t stream);
 
+/*
+ * Sink4/local128 BF16 protection (App. C.5, "BF16 protection and cache
+ * lifecycle"). For a request of L cached tokens the protected positions are
+ *     P_L = {0, ..., min(4, L) - 1}  U  {max(0, L - 128), ..., L - 1};
+ * attention reads their pre-quantisation bf16 content and RoPE-key values and
+ * reads every other position from the packed cache, all under one softmax. A
+ * packed copy is written for every token, protected or not, so a token leaving
+ * the recent window switches to its packed copy with no further work.
+ *
+ * Protection buffer (caller-owned, one per request): [num_seqs][132][576] bf16,
+ * qmla_protect_bytes_per_seq() = 132 * 576 * 2 = 152064 bytes per request (the
+ * paper's figure), 16-byte aligned. A row holds a token's 512 latent values
+ * then its 64 RoPE-key values; rows 0..3 hold sink positions 0..3, row
+ * 4 + (p mod 128) holds recent position p. The buffer needs no initialisation:
+ * a row is only read once the writer has filled it.
+ */
+size_t qmla_protect_bytes_per_seq(void);
+
+/* qmla_quant_append plus the protection rows: token i (request s = seq_ids[i],
+ * position p) is also copied into row p when p < 4 and into row 4 + (p mod 128)
+ * when p >= seq_lens_dev[s] - 128, where seq_lens_dev [num_seqs] int32 holds the
+ * requests' lengths after this call. So one call may carry a whole prefill:
+ * positions older than the recent window never reach the ring, and no two
+ * positions of one call share a row. latent_dev, k_pe_dev and prot_dev must be
+ * 16-byte aligned; the other arguments and errors are those of qmla_quant_append. */
+int qmla_quant_append_protected(void* pool_dev, int c_bits, int num_blocks, const uint16_t* latent_dev,
+                                const uint16_t* k_pe_dev, const int32_t* seq_ids_dev,
+                                const int32_t* positions_dev, int n, const int32_t* block_table_dev,
+                                int num_seqs, int max_blocks, const int32_t* seq_lens_dev, void* prot_dev,
+                                uint32_t* dev_err_dev, qmla_stream_t stream);
+
 /* Workspace bytes qmla_mla_decode needs for this batch and head count on the
  * current device (split plan + split partials). */
 size_t qmla_decode_workspace_bytes(int batch, int heads);
@@ -148,6 +179,19 @@ int qmla_mla_decode(const void* pool_dev, int c_bits, int num_blocks, const uint
                     int max_blocks, const int32_t* seq_lens_dev, float softmax_scale,
                     float* out_dev, float* lse_dev, void* workspace_dev, size_t workspace_bytes,
                     uint32_t* dev_err_dev, qmla_stream_t stream);
+
+/* qmla_mla_decode under sink4/local128 protection: for request b with
+ * L = seq_lens_dev[b], positions in P_L read row p (p < 4) or row 4 + (p mod 128)
+ * of prot_dev[b] (rounded to fp16 like the BF16 cache path), every other
+ * position the packed cache; one global softmax over all L positions. The
+ * buffer must hold every protected position (qmla_quant_append_protected with
+ * the same lengths leaves it so). prot_dev 16-byte aligned, non-null; outputs,
+ * workspace and errors as qmla_mla_decode. */
+int qmla_mla_decode_protected(const void* pool_dev, int c_bits, int num_blocks, const uint16_t* q_latent_dev,
+                              const uint16_t* q_pe_dev, int batch, int heads, const int32_t* block_table_dev,
+                              int max_blocks, const int32_t* seq_lens_dev, const void* prot_dev,
+                              float softmax_scale, float* out_dev, float* lse_dev, void* workspace_dev,
+                              size_t workspace_bytes, uint32_t* dev_err_dev, qmla_stream_t stream);
 
 /* The same decode over the BF16 comparison cache (same kernel, no dequantisation;
  * the paper's BF16 baseline, App. F.1). */

@@ -67,6 +67,12 @@ def lib():
     L.qmla_static_scratch_bytes.argtypes, L.qmla_static_scratch_bytes.restype = [], sz
     L.qmla_mla_decode_static.argtypes = [vp, i32, i32, vp, vp, i32, i32, vp, i32, vp, f32, vp, vp, vp, vp]
     L.qmla_mla_decode_static.restype = i32
+    L.qmla_protect_bytes_per_seq.argtypes, L.qmla_protect_bytes_per_seq.restype = [], sz
+    L.qmla_quant_append_protected.argtypes = [vp, i32, i32, vp, vp, vp, vp, i32, vp, i32, i32, vp, vp, vp, vp]
+    L.qmla_quant_append_protected.restype = i32
+    L.qmla_mla_decode_protected.argtypes = [vp, i32, i32, vp, vp, i32, i32, vp, i32, vp, vp, f32, vp, vp, vp, sz,
+                                            vp, vp]
+    L.qmla_mla_decode_protected.restype = i32
     _lib = L
     return L
 
@@ -118,6 +124,23 @@ def quant_append(pool: torch.Tensor, c_bits: int, latent: torch.Tensor, k_pe: to
     _check("qmla_quant_append", st)
 
 
+def protect_bytes_per_seq() -> int:
+    return int(lib().qmla_protect_bytes_per_seq())
+
+
+def quant_append_protected(pool: torch.Tensor, c_bits: int, latent: torch.Tensor, k_pe: torch.Tensor,
+                           seq_ids: torch.Tensor | None, positions: torch.Tensor, block_table: torch.Tensor,
+                           seq_lens: torch.Tensor, prot: torch.Tensor, dev_err: torch.Tensor, stream=None) -> None:
+    """qmla_quant_append_protected: quant_append plus the sink/recent bf16 rows;
+    seq_lens int32 [S] = lengths after this call; prot [S, 132, 576] bf16."""
+    n = latent.shape[0]
+    st = lib().qmla_quant_append_protected(_ptr(pool), c_bits, pool.shape[0], _ptr(latent), _ptr(k_pe),
+                                           _ptr(seq_ids), _ptr(positions), n, _ptr(block_table),
+                                           block_table.shape[0], block_table.shape[1], _ptr(seq_lens), _ptr(prot),
+                                           _ptr(dev_err), _stream(stream))
+    _check("qmla_quant_append_protected", st)
+
+
 def bf16_append(pool: torch.Tensor, latent: torch.Tensor, k_pe: torch.Tensor, seq_ids: torch.Tensor | None,
                 positions: torch.Tensor, block_table: torch.Tensor, dev_err: torch.Tensor, stream=None) -> None:
     n = latent.shape[0]
@@ -137,6 +160,20 @@ def mla_decode(pool: torch.Tensor, c_bits: int, q_latent: torch.Tensor, q_pe: to
                                _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel() * workspace.element_size(),
                                _ptr(dev_err), _stream(stream))
     _check("qmla_mla_decode", st)
+
+
+def mla_decode_protected(pool: torch.Tensor, c_bits: int, q_latent: torch.Tensor, q_pe: torch.Tensor,
+                         block_table: torch.Tensor, seq_lens: torch.Tensor, prot: torch.Tensor, softmax_scale: float,
+                         out: torch.Tensor, lse: torch.Tensor | None, workspace: torch.Tensor, dev_err: torch.Tensor,
+                         stream=None) -> None:
+    """qmla_mla_decode_protected: mla_decode with sink4/local128 bf16 rows from prot [B, 132, 576]."""
+    B, H = q_latent.shape[0], q_latent.shape[1]
+    st = lib().qmla_mla_decode_protected(_ptr(pool), c_bits, pool.shape[0], _ptr(q_latent), _ptr(q_pe), B, H,
+                                         _ptr(block_table), block_table.shape[1], _ptr(seq_lens), _ptr(prot),
+                                         float(softmax_scale), _ptr(out), _ptr(lse), _ptr(workspace),
+                                         workspace.numel() * workspace.element_size(), _ptr(dev_err),
+                                         _stream(stream))
+    _check("qmla_mla_decode_protected", st)
 
 
 def mla_decode_bf16cache(pool: torch.Tensor, q_latent: torch.Tensor, q_pe: torch.Tensor, block_table: torch.Tensor,

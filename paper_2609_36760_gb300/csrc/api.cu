@@ -62,10 +62,11 @@ int append_common_checks(const void* pool, int num_blocks, const uint16_t* laten
 int decode_common(const void* pool, int kind, int num_blocks, const uint16_t* q_latent, const uint16_t* q_pe,
                   int batch, int heads, const int32_t* table, int max_blocks, const int32_t* seq_lens,
                   float softmax_scale, float* out, float* lse, void* workspace, size_t workspace_bytes,
-                  uint32_t* dev_err, qmla_stream_t stream) {
+                  uint32_t* dev_err, qmla_stream_t stream, const void* prot = nullptr) {
   if (pool == nullptr || q_latent == nullptr || q_pe == nullptr || table == nullptr || seq_lens == nullptr ||
       out == nullptr || workspace == nullptr)
     return QMLA_ERR_INVALID_ARG;
+  if (prot != nullptr && !aligned(prot, 16)) return QMLA_ERR_INVALID_ARG;
   if (batch <= 0 || heads < 1 || heads > 128 || num_blocks <= 0 || max_blocks <= 0) return QMLA_ERR_INVALID_ARG;
   if (!(softmax_scale > 0.0f) || softmax_scale > 1e30f) return QMLA_ERR_INVALID_ARG;
   if (!aligned(pool, 16) || !aligned(q_latent, 16) || !aligned(q_pe, 16) || !aligned(table, 4) ||
@@ -95,6 +96,7 @@ int decode_common(const void* pool, int kind, int num_blocks, const uint16_t* q_
   a.workspace = workspace;
   a.dev_err = dev_err;
   a.grid = di.sms;
+  a.prot = prot;
   a.ev_before_main = g_ev_before_main;
   a.ev_after_main = g_ev_after_main;
   cudaError_t e = qmla::launch_decode(a, reinterpret_cast<cudaStream_t>(stream));
@@ -133,6 +135,30 @@ int qmla_quant_append(void* pool_dev, int c_bits, int num_blocks, const uint16_t
   return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
 }
 
+size_t qmla_protect_bytes_per_seq(void) { return static_cast<size_t>(qmla::kProtRows) * qmla::kDqk * 2; }
+
+int qmla_quant_append_protected(void* pool_dev, int c_bits, int num_blocks, const uint16_t* latent_dev,
+                                const uint16_t* k_pe_dev, const int32_t* seq_ids_dev,
+                                const int32_t* positions_dev, int n, const int32_t* block_table_dev,
+                                int num_seqs, int max_blocks, const int32_t* seq_lens_dev, void* prot_dev,
+                                uint32_t* dev_err_dev, qmla_stream_t stream) {
+  if (c_bits != 4 && c_bits != 2) return QMLA_ERR_INVALID_ARG;
+  int st = append_common_checks(pool_dev, num_blocks, latent_dev, k_pe_dev, positions_dev, n, block_table_dev,
+                                num_seqs, max_blocks);
+  if (st != QMLA_OK) return st;
+  if (prot_dev == nullptr || seq_lens_dev == nullptr || !aligned(prot_dev, 16) || !aligned(seq_lens_dev, 4) ||
+      !aligned(latent_dev, 16) || !aligned(k_pe_dev, 16))
+    return QMLA_ERR_INVALID_ARG;
+  if (n == 0) return QMLA_OK;
+  DevInfo di;
+  if ((st = current_device_info(di)) != QMLA_OK) return st;
+  cudaError_t e = qmla::launch_quant_append(pool_dev, c_bits, num_blocks, latent_dev, k_pe_dev, seq_ids_dev,
+                                            positions_dev, n, block_table_dev, num_seqs, max_blocks,
+                                            dev_err_dev, reinterpret_cast<cudaStream_t>(stream), prot_dev,
+                                            seq_lens_dev);
+  return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
+}
+
 int qmla_bf16_append(void* pool_dev, int num_blocks, const uint16_t* latent_dev, const uint16_t* k_pe_dev,
                      const int32_t* seq_ids_dev, const int32_t* positions_dev, int n,
                      const int32_t* block_table_dev, int num_seqs, int max_blocks, uint32_t* dev_err_dev,
@@ -163,6 +189,18 @@ int qmla_mla_decode(const void* pool_dev, int c_bits, int num_blocks, const uint
   return decode_common(pool_dev, c_bits, num_blocks, q_latent_dev, q_pe_dev, batch, heads, block_table_dev,
                        max_blocks, seq_lens_dev, softmax_scale, out_dev, lse_dev, workspace_dev, workspace_bytes,
                        dev_err_dev, stream);
+}
+
+int qmla_mla_decode_protected(const void* pool_dev, int c_bits, int num_blocks, const uint16_t* q_latent_dev,
+                              const uint16_t* q_pe_dev, int batch, int heads, const int32_t* block_table_dev,
+                              int max_blocks, const int32_t* seq_lens_dev, const void* prot_dev,
+                              float softmax_scale, float* out_dev, float* lse_dev, void* workspace_dev,
+                              size_t workspace_bytes, uint32_t* dev_err_dev, qmla_stream_t stream) {
+  if (c_bits != 4 && c_bits != 2) return QMLA_ERR_INVALID_ARG;
+  if (prot_dev == nullptr) return QMLA_ERR_INVALID_ARG;
+  return decode_common(pool_dev, c_bits, num_blocks, q_latent_dev, q_pe_dev, batch, heads, block_table_dev,
+                       max_blocks, seq_lens_dev, softmax_scale, out_dev, lse_dev, workspace_dev, workspace_bytes,
+                       dev_err_dev, stream, prot_dev);
 }
 
 int qmla_mla_decode_bf16cache(const void* pool_dev, int num_blocks, const uint16_t* q_latent_dev,

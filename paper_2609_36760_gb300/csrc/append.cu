@@ -67,12 +67,38 @@ __device__ __forceinline__ uint8_t* token_block(uint8_t* pool, size_t block_byte
   return pool + static_cast<size_t>(blk) * block_bytes;
 }
 
+// Sink/recent BF16 protection rows (App. C.5, "BF16 protection and cache
+// lifecycle"): position p of a request whose length after this write is L goes
+// to row p when p < 4 and to row 4 + p mod 128 when p >= L - 128. The warp
+// copies the token's 576 bf16 values (1152 bytes) as 16-byte vectors.
+__device__ __forceinline__ void protect_row(uint4* prot, const uint4* latent, const uint4* k_pe, int tok, int seq,
+                                            int pos, int L, int lane) {
+  uint4* base = prot + static_cast<size_t>(seq) * kProtRows * (kDqk * 2 / 16);
+  const uint4* lat = latent + static_cast<size_t>(tok) * (kDc * 2 / 16);  // 64 vectors
+  const uint4* kp = k_pe + static_cast<size_t>(tok) * (kDr * 2 / 16);     // 8 vectors
+  const uint4 a = lat[lane], b = lat[32 + lane];
+  const uint4 c = lane < 8 ? kp[lane] : make_uint4(0, 0, 0, 0);
+#pragma unroll
+  for (int which = 0; which < 2; ++which) {
+    int row = -1;
+    if (which == 0 && pos < kSinkTokens) row = pos;
+    if (which == 1 && pos >= L - kRecentTokens) row = kSinkTokens + pos % kRecentTokens;
+    if (row < 0) continue;
+    uint4* dst = base + static_cast<size_t>(row) * (kDqk * 2 / 16);
+    dst[lane] = a;
+    dst[32 + lane] = b;
+    if (lane < 8) dst[64 + lane] = c;
+  }
+}
+
+// prot / lens: the protection buffer [num_seqs][132][576] bf16 and the
+// requests' lengths after this write, or null for an unprotected cache.
 template <int CB>
 __global__ void __launch_bounds__(256) quant_append_kernel(
     uint8_t* __restrict__ pool, int num_blocks, const __nv_bfloat162* __restrict__ latent,
     const __nv_bfloat162* __restrict__ k_pe, const int32_t* __restrict__ seq_ids,
     const int32_t* __restrict__ positions, int n, const int32_t* __restrict__ table, int num_seqs,
-    int max_blocks, uint32_t* dev_err) {
+    int max_blocks, uint32_t* dev_err, uint4* __restrict__ prot, const int32_t* __restrict__ lens) {
   using L = BlockLayout<CB>;
   const int tok = static_cast<int>((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
   const int lane = threadIdx.x & 31;
@@ -81,6 +107,11 @@ __global__ void __launch_bounds__(256) quant_append_kernel(
   uint8_t* blk = token_block(pool, L::kBytes, num_blocks, seq_ids, positions, tok, table, num_seqs,
                              max_blocks, lane == 0 ? dev_err : nullptr, slot);
   if (blk == nullptr) return;
+  if (prot != nullptr) {
+    const int seq = seq_ids != nullptr ? seq_ids[tok] : tok;
+    protect_row(prot, reinterpret_cast<const uint4*>(latent), reinterpret_cast<const uint4*>(k_pe), tok, seq,
+                positions[tok], lens[seq], lane);
+  }
 
 #pragma unroll 1
   for (int g = 0; g < kGroups; ++g) {
@@ -131,7 +162,8 @@ __global__ void __launch_bounds__(256) bf16_append_kernel(
 cudaError_t launch_quant_append(void* pool, int c_bits, int num_blocks, const uint16_t* latent,
                                 const uint16_t* k_pe, const int32_t* seq_ids,
                                 const int32_t* positions, int n, const int32_t* table, int num_seqs,
-                                int max_blocks, uint32_t* dev_err, cudaStream_t stream) {
+                                int max_blocks, uint32_t* dev_err, cudaStream_t stream, void* prot,
+                                const int32_t* lens) {
   if (n == 0) return cudaSuccess;
   const dim3 block(256);
   const dim3 grid(static_cast<unsigned>((static_cast<long long>(n) * 32 + 255) / 256));
@@ -140,11 +172,11 @@ cudaError_t launch_quant_append(void* pool, int c_bits, int num_blocks, const ui
   if (c_bits == 4) {
     quant_append_kernel<4><<<grid, block, 0, stream>>>(static_cast<uint8_t*>(pool), num_blocks, lat,
                                                        kp, seq_ids, positions, n, table, num_seqs,
-                                                       max_blocks, dev_err);
+                                                       max_blocks, dev_err, static_cast<uint4*>(prot), lens);
   } else {
     quant_append_kernel<2><<<grid, block, 0, stream>>>(static_cast<uint8_t*>(pool), num_blocks, lat,
                                                        kp, seq_ids, positions, n, table, num_seqs,
-                                                       max_blocks, dev_err);
+                                                       max_blocks, dev_err, static_cast<uint4*>(prot), lens);
   }
   return cudaGetLastError();
 }

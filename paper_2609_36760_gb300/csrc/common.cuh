@@ -15,6 +15,10 @@ constexpr int kGroup = 64;         // quantisation group (App. C.4)
 constexpr int kGroups = 9;         // 8 content groups + 1 RoPE-key group
 constexpr int kBlockTokens = 64;   // tokens per cache block (page)
 constexpr int kPeBits = 4;         // RoPE key bit width
+// sink4/local128 protection buffer: rows 0..3 sink positions, 4 + p mod 128 recent p.
+constexpr int kSinkTokens = 4;
+constexpr int kRecentTokens = 128;
+constexpr int kProtRows = kSinkTokens + kRecentTokens;
 
 // Block layout for content bit width CB (see include/qmla.h).
 template <int CB>

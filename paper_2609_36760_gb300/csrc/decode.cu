@@ -83,6 +83,8 @@ constexpr int kTraceCtas = 8, kTraceEvents = 128, kTraceTiles = 32;
 
 struct Params {
   const uint8_t* pool;
+  // sink4/local128 protection buffer [batch][132][576] bf16, or null (unprotected).
+  const uint8_t* prot;
   int num_blocks;
   const __nv_bfloat16* q_lat;
   const __nv_bfloat16* q_pe;
@@ -308,7 +310,7 @@ struct Fetch {
 // The table column is clamped so that rows past the sequence end never read
 // beyond the sequence's table row.
 struct RowRef {
-  int entry, len, j;
+  int entry, len, j, b;
   bool has;
 };
 __device__ __forceinline__ RowRef row_ref(const Params& p, const Sched& s, int row) {
@@ -317,8 +319,10 @@ __device__ __forceinline__ RowRef row_ref(const Params& p, const Sched& s, int r
   r.entry = -1;
   r.len = 0;
   r.j = 0;
+  r.b = 0;
   if (!r.has) return r;
   const int b = s.u / p.n_hg;
+  r.b = b;
   r.j = s.t - s.pu0;
   r.len = p.seq_lens[b];
   const int lb = min(2 * r.j + (row >> 6), p.max_blocks - 1);
@@ -336,6 +340,26 @@ __device__ __forceinline__ const uint8_t* resolve_row(const Params& p, const Row
   valid = true;
   constexpr size_t kBlk = CB == 16 ? static_cast<size_t>(kBf16BlockBytes) : BlockLayout<CB == 16 ? 4 : CB>::kBytes;
   return p.pool + static_cast<size_t>(r.entry) * kBlk;
+}
+
+// The protection-buffer row a tile row attends with (App. C.5, "BF16
+// protection and cache lifecycle": position p of a length-L request is
+// protected iff p < min(4, L) or p >= L - 128), or null when the row is read
+// from the packed cache. Sink positions read their sink row, which the writer
+// always fills; recent ones the ring row 4 + p mod 128.
+__device__ __forceinline__ const uint8_t* prot_row(const Params& p, const RowRef& r, int row) {
+  if (p.prot == nullptr || !r.has) return nullptr;
+  const int pos = kTileTokens * r.j + row;
+  if (pos >= r.len) return nullptr;
+  int pr;
+  if (pos < kSinkTokens) {
+    pr = pos;
+  } else if (pos >= r.len - kRecentTokens) {
+    pr = kSinkTokens + pos % kRecentTokens;
+  } else {
+    return nullptr;
+  }
+  return p.prot + (static_cast<size_t>(r.b) * kProtRows + pr) * (kDqk * 2);
 }
 
 template <int CB>
@@ -395,6 +419,32 @@ __device__ __forceinline__ void store_row(uint32_t chunk_base, int row, const Fe
              dq2(__byte_perm(c1, K, 0x4342), zz, ss), dq2(__byte_perm(c2, K, 0x4342), zz, ss),
              dq2(__byte_perm(c3, K, 0x4342), zz, ss));
     }
+  }
+}
+
+// A protected row's chunk k: 64 bf16 values (8 x 16 bytes) rounded to fp16 and
+// placed in the same within-piece channel order as the packed rows
+// (bf16 -> fp16 is exact for magnitudes in [2^-14, 65504]).
+template <int CB>
+__device__ __forceinline__ void store_row_prot(uint32_t chunk_base, int row, const uint4 (&v)[8], int k) {
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const uint32_t w[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+    float f[8];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      f[2 * e] = bf16_lo(w[e]);
+      f[2 * e + 1] = bf16_hi(w[e]);
+    }
+    uint32_t o[4];
+    if (k < 8) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) o[e] = pack_h2(f[Perm<CB>::at(2 * e)], f[Perm<CB>::at(2 * e + 1)]);
+    } else {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) o[e] = pack_h2(f[Perm<4>::at(2 * e)], f[Perm<4>::at(2 * e + 1)]);
+    }
+    sts_v4(chunk_base + swz_off(row, i, 128), o[0], o[1], o[2], o[3]);
   }
 }
 
@@ -665,8 +715,11 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     ref0.entry = row < 64 ? fr.x : fr.y;
     ref0.len = fr.z;
     ref0.j = fr.w;
+    ref0.b = sc.u / p.n_hg;
   }
-  const uint8_t* blk_cur = resolve_row<CB>(p, ref0, row, valid_cur);
+  // A protected row reads its BF16 row instead of the packed cache.
+  const uint8_t* psrc_cur = prot_row(p, ref0, row);
+  const uint8_t* blk_cur = psrc_cur != nullptr ? nullptr : resolve_row<CB>(p, ref0, row, valid_cur);
   if constexpr (CB != 16) {
 #pragma unroll
     for (int kc = 0; kc < kMyChunks; ++kc) {
@@ -689,7 +742,8 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     // The next tile's block pointer (its table entry was loaded a tile ago)
     // and the table entry of the tile after it.
     bool valid_nx = false;
-    const uint8_t* blk_nx = resolve_row<CB>(p, ref_nx, row, valid_nx);
+    const uint8_t* psrc_nx = prot_row(p, ref_nx, row);
+    const uint8_t* blk_nx = psrc_nx != nullptr ? nullptr : resolve_row<CB>(p, ref_nx, row, valid_nx);
     Sched nn = nx;
     nn.next();
     const RowRef ref_nn = row_ref(p, nn, row);
@@ -700,6 +754,13 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     for (int kc = 0; kc < kMyChunks; ++kc) {
       const int k = 2 * kc + par;
       if (k >= kNumChunks) break;
+      uint4 pv[CB == 16 ? 1 : 8];  // a protected row's chunk, loaded before the slot wait
+      if constexpr (CB != 16) {
+        if (psrc_cur != nullptr) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) pv[i] = ldg_nc_v4(psrc_cur + k * 128 + i * 16);
+        }
+      }
       if (!(ok = wwait(slot_bar(ctl, k), (it & 1u) ^ 1u, ctl, kSiteDqSlot, p.dev_err))) break;
       if (lane == 0) QMLA_TRACE(88 + warp, it);  // (overwritten per chunk: last slot wait)
       if constexpr (CB == 16) {
@@ -718,7 +779,11 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
 #pragma unroll
         for (int i = 0; i < 8; ++i) cur[i] = nxt[i];
       } else {
-        store_row<CB>(chunks + k * kChunkBytes, row, f[kc], CB == 4 || k == 8);
+        if (psrc_cur != nullptr) {
+          store_row_prot<CB>(chunks + k * kChunkBytes, row, pv, k);
+        } else {
+          store_row<CB>(chunks + k * kChunkBytes, row, f[kc], CB == 4 || k == 8);
+        }
         f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);  // the next tile's rows of this chunk
       }
       fence_proxy_async_smem();
@@ -730,6 +795,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     if (lane == 0) QMLA_TRACE(32 + warp, it);
     blk_cur = blk_nx;
     valid_cur = valid_nx;
+    psrc_cur = psrc_nx;
     nx = nn;
     ref_nx = ref_nn;
     const TileInfo ti = tile_info(sc, p);  // ntok of this tile for the softmax (loaded long ago)
@@ -1222,6 +1288,7 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
   uint8_t* ws = static_cast<uint8_t*>(a.workspace);
   Params prm;
   prm.pool = static_cast<const uint8_t*>(a.pool);
+  prm.prot = a.cache_kind == 16 ? nullptr : static_cast<const uint8_t*>(a.prot);
   prm.num_blocks = a.num_blocks;
   prm.q_lat = reinterpret_cast<const __nv_bfloat16*>(a.q_latent);
   prm.q_pe = reinterpret_cast<const __nv_bfloat16*>(a.q_pe);

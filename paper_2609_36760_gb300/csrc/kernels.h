@@ -9,7 +9,8 @@ namespace qmla {
 cudaError_t launch_quant_append(void* pool, int c_bits, int num_blocks, const uint16_t* latent,
                                 const uint16_t* k_pe, const int32_t* seq_ids,
                                 const int32_t* positions, int n, const int32_t* table, int num_seqs,
-                                int max_blocks, uint32_t* dev_err, cudaStream_t stream);
+                                int max_blocks, uint32_t* dev_err, cudaStream_t stream,
+                                void* prot = nullptr, const int32_t* lens = nullptr);
 
 cudaError_t launch_bf16_append(void* pool, int num_blocks, const uint16_t* latent,
                                const uint16_t* k_pe, const int32_t* seq_ids,
@@ -41,6 +42,7 @@ struct DecodeArgs {
   void* workspace;
   uint32_t* dev_err;
   int grid;  // CTAs of the main kernel (one per SM)
+  const void* prot = nullptr;  // sink4/local128 protection buffer, or null
   cudaEvent_t ev_before_main = nullptr;  // optional, recorded around the main kernel
   cudaEvent_t ev_after_main = nullptr;
 };

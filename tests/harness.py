@@ -13,6 +13,7 @@ import torch
 import paper_2609_36760_gb300 as Q
 from oracle import attention as OA
 from oracle import layout as OL
+from oracle import protection as OP
 from oracle import quantizer as OQ
 from workloads import synthetic as W
 
@@ -29,9 +30,10 @@ def rel_l2(a, b) -> float:
 class Case:
     """A workload materialised on the GPU (packed or BF16 cache) plus its inputs on the host."""
 
-    def __init__(self, w: W.Workload, bf16_cache: bool = False, device: str = "cuda"):
+    def __init__(self, w: W.Workload, bf16_cache: bool = False, device: str = "cuda", protect: bool = False):
         self.w = w
         self.bf16 = bf16_cache
+        self.protect = protect
         self.dev = device
         self.prefill = W.seq_lengths(w)
         self.final = W.final_lengths(w)
@@ -44,6 +46,10 @@ class Case:
         self.table_d = table.to(device)
         self.dev_err = torch.zeros(1, dtype=torch.int32, device=device)
         self._tok = {}
+        # sink4/local128 protection rows, poisoned with bf16 NaN so that a row read
+        # before the writer filled it shows up in the output
+        self.prot = (torch.full((w.batch, 132, 576), 0xFFFF, dtype=torch.int32, device=device)
+                     .to(torch.int16).view(torch.bfloat16) if protect else None)
 
     # host-side inputs, cached per sequence (bf16 tensors up to the final length)
     def tokens(self, b: int):
@@ -52,12 +58,16 @@ class Case:
             self._tok[b] = (W.latent_for_seq(self.w, b, n, self.gains), W.kpe_for_seq(self.w, b, n))
         return self._tok[b]
 
-    def append(self, lat: torch.Tensor, kpe: torch.Tensor, seq_ids, positions) -> None:
+    def append(self, lat: torch.Tensor, kpe: torch.Tensor, seq_ids, positions, lens_after=None) -> None:
         lat_d = lat.contiguous().to(self.dev)
         kpe_d = kpe.contiguous().to(self.dev)
         sid = None if seq_ids is None else torch.as_tensor(seq_ids, dtype=torch.int32).to(self.dev)
         pos = torch.as_tensor(positions, dtype=torch.int32).to(self.dev)
-        if self.bf16:
+        if self.protect:
+            la = torch.as_tensor(lens_after, dtype=torch.int32).to(self.dev)
+            Q.quant_append_protected(self.pool, self.w.c_bits, lat_d, kpe_d, sid, pos, self.table_d, la, self.prot,
+                                     self.dev_err)
+        elif self.bf16:
             Q.bf16_append(self.pool, lat_d, kpe_d, sid, pos, self.table_d, self.dev_err)
         else:
             Q.quant_append(self.pool, self.w.c_bits, lat_d, kpe_d, sid, pos, self.table_d, self.dev_err)
@@ -75,10 +85,10 @@ class Case:
             sids.append(torch.full((n,), b, dtype=torch.int32)); poss.append(torch.arange(n, dtype=torch.int32))
             pending += n
             if pending >= chunk_tokens:
-                self.append(torch.cat(lats), torch.cat(kps), torch.cat(sids), torch.cat(poss))
+                self.append(torch.cat(lats), torch.cat(kps), torch.cat(sids), torch.cat(poss), self.prefill)
                 lats, kps, sids, poss, pending = [], [], [], [], 0
         if pending:
-            self.append(torch.cat(lats), torch.cat(kps), torch.cat(sids), torch.cat(poss))
+            self.append(torch.cat(lats), torch.cat(kps), torch.cat(sids), torch.cat(poss), self.prefill)
 
     def lengths_at(self, step: int) -> list[int]:
         return [n + self.w.append * (step + 1) for n in self.prefill]
@@ -94,7 +104,7 @@ class Case:
             for k in range(self.w.append):
                 lats.append(lat[a0 + k:a0 + k + 1]); kps.append(kp[a0 + k:a0 + k + 1])
                 sids.append(b); poss.append(a0 + k)
-        self.append(torch.cat(lats), torch.cat(kps), sids, poss)
+        self.append(torch.cat(lats), torch.cat(kps), sids, poss, self.lengths_at(step))
 
     def decode(self, step: int, lens: list[int] | None = None, queries=None):
         ql, qp = queries if queries is not None else W.queries(self.w, step)
@@ -106,7 +116,10 @@ class Case:
         ws.fill_(0x7F)
         sl = torch.tensor(lens, dtype=torch.int32, device=self.dev)
         ql_d, qp_d = ql.contiguous().to(self.dev), qp.contiguous().to(self.dev)
-        if self.bf16:
+        if self.protect:
+            Q.mla_decode_protected(self.pool, self.w.c_bits, ql_d, qp_d, self.table_d, sl, self.prot, TAU, out, lse,
+                                   ws, self.dev_err)
+        elif self.bf16:
             Q.mla_decode_bf16cache(self.pool, ql_d, qp_d, self.table_d, sl, TAU, out, lse, ws, self.dev_err)
         else:
             Q.mla_decode(self.pool, self.w.c_bits, ql_d, qp_d, self.table_d, sl, TAU, out, lse, ws, self.dev_err)
@@ -126,8 +139,18 @@ class Case:
         q, s, z = OL.quantize_tokens(latf, kpf, self.w.c_bits)
         if fp16_tiles:
             x = OQ.dequantize_fp16(q.reshape(L, 9, 64), s, z).astype(np.float64).reshape(L, 576)
-            return x[:, :512], x[:, 512:]
-        return OA.dequantize_tokens(q, s, z)
+            C, K = x[:, :512], x[:, 512:]
+        else:
+            C, K = OA.dequantize_tokens(q, s, z)
+        if self.protect:
+            # protected positions attend with the original values (rounded to fp16
+            # in the tile-exact variant, as the kernel's tiles hold them)
+            C, K = np.array(C), np.array(K)
+            P = OP.protected_positions(L)
+            rnd = (lambda a: a.astype(np.float16).astype(np.float64)) if fp16_tiles else (lambda a: a)
+            C[P] = rnd(latf[P])
+            K[P] = rnd(kpf[P])
+        return C, K
 
     def oracle_decode(self, b: int, L: int, step: int = 0, heads=None, fp16_tiles: bool = False, queries=None):
         ql, qp = queries if queries is not None else W.queries(self.w, step)
@@ -146,3 +169,10 @@ class Case:
                             np.full(n, b), np.arange(n), self.table.numpy())
         blocks = sorted({int(x) for b in seqs for x in self.table[b].tolist() if x >= 0})
         return blocks, pool[blocks]
+
+    def oracle_prot_rows(self, b: int, L: int) -> np.ndarray:
+        """Expected protection rows of request b at length L: [132, 576] fp64, NaN where unused."""
+        lat, kp = self.tokens(b)
+        buf = np.full((1, 132, 576), np.nan)
+        OP.write_protection(buf, lat[:L].double().numpy(), kp[:L].double().numpy(), np.zeros(L, int), np.arange(L), [L])
+        return buf[0]
