@@ -47,6 +47,8 @@ def parse():
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(W.WORKLOADS))
     ap.add_argument("--bf16-cache", action="store_true", help="decode the BF16 comparison cache instead")
+    ap.add_argument("--protect", action="store_true",
+                    help="sink4/local128 BF16 protection (the paper's C4R4 serving configuration)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
@@ -154,16 +156,20 @@ def decode_cu_hash() -> str:
 class Workspace:
     """GPU state of one workload: pool, block table, per-step inputs."""
 
-    def __init__(self, w: W.Workload, bf16: bool, dev: torch.device, nsteps: int):
+    def __init__(self, w: W.Workload, bf16: bool, dev: torch.device, nsteps: int, protect: bool = False):
         import paper_2609_36760_gb300 as Q
         self.Q = Q
         self.w, self.bf16, self.dev = w, bf16, dev
+        self.protect = protect and not bf16
         self.prefill = W.seq_lengths(w)
         table, nblocks = W.block_table(w)
         self.table = table.to(dev)
         bb = Q.bf16_block_bytes() if bf16 else Q.block_bytes(w.c_bits)
         self.pool = torch.zeros((nblocks, bb), dtype=torch.uint8, device=dev)
         self.err = torch.zeros(1, dtype=torch.int32, device=dev)
+        # per-request 132 x 576 bf16 protection rows (152,064 bytes each)
+        self.prot = (torch.zeros((w.batch, 132, 576), dtype=torch.bfloat16, device=dev) if self.protect else None)
+        self.prefill_lens = torch.tensor(self.prefill, dtype=torch.int32, device=dev)
         gains = W.channel_gains(w)
         self.nsteps = max(1, min(nsteps, w.steps))
         self.step_in = [dict(lat=[], kp=[], pos=[]) for _ in range(self.nsteps)]
@@ -174,7 +180,7 @@ class Workspace:
             kp = W.kpe_for_seq(w, b, n_all)
             n = self.prefill[b]
             self._append(lat[:n].to(dev), kp[:n].to(dev), torch.full((n,), b, dtype=torch.int32, device=dev),
-                         torch.arange(n, dtype=torch.int32, device=dev))
+                         torch.arange(n, dtype=torch.int32, device=dev), self.prefill_lens)
             for s in range(self.nsteps):
                 for k in range(w.append):
                     p = n + w.append * s + k
@@ -200,10 +206,13 @@ class Workspace:
         self.lse = torch.empty((w.batch, w.heads), dtype=torch.float32, device=dev)
         self.ws = Q.workspace_for(w.batch, w.heads, dev)
 
-    def _append(self, lat, kp, sid, pos):
+    def _append(self, lat, kp, sid, pos, lens_after=None):
         if lat.shape[0] == 0:
             return
-        if self.bf16:
+        if self.protect:
+            self.Q.quant_append_protected(self.pool, self.w.c_bits, lat, kp, sid, pos, self.table, lens_after,
+                                          self.prot, self.err)
+        elif self.bf16:
             self.Q.bf16_append(self.pool, lat, kp, sid, pos, self.table, self.err)
         else:
             self.Q.quant_append(self.pool, self.w.c_bits, lat, kp, sid, pos, self.table, self.err)
@@ -212,8 +221,11 @@ class Workspace:
         d = d if d is not None else self.steps[s % self.nsteps]["dev"]
         out = self.out if out is None else out
         lse = self.lse if lse is None else lse
-        self._append(d["lat"], d["kp"], d["sid"], d["pos"])
-        if self.bf16:
+        self._append(d["lat"], d["kp"], d["sid"], d["pos"], d["lens"])
+        if self.protect:
+            self.Q.mla_decode_protected(self.pool, self.w.c_bits, d["ql"], d["qp"], self.table, d["lens"], self.prot,
+                                        TAU, out, lse, self.ws, self.err)
+        elif self.bf16:
             self.Q.mla_decode_bf16cache(self.pool, d["ql"], d["qp"], self.table, d["lens"], TAU, out, lse, self.ws,
                                         self.err)
         else:
@@ -235,7 +247,7 @@ def run_native(args, ws_world: int, rank: int, local: int):
         dist.init_process_group("nccl", device_id=dev)
     w = W.WORKLOADS[args.workload]
     K, Wm = args.steps, args.warmup
-    state = Workspace(w, args.bf16_cache, dev, K + Wm)
+    state = Workspace(w, args.bf16_cache, dev, K + Wm, protect=args.protect)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # larger than the 126 MB L2
     stream = torch.cuda.current_stream(dev)
 
@@ -325,7 +337,8 @@ def run_native(args, ws_world: int, rank: int, local: int):
         "ms_per_step": round(ms_step_max, 5), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "f16", "data": "synthetic (seeded generators, workloads/synthetic.py)",
         "config": {"workload": w.name, "batch_per_gpu": w.batch, "heads": w.heads, "c_bits": w.c_bits,
-                   "pe_bits": 4, "cache": "bf16" if args.bf16_cache else f"int{w.c_bits}/int4 packed",
+                   "pe_bits": 4, "cache": "bf16" if args.bf16_cache else (
+                       f"int{w.c_bits}/int4 packed" + (" + sink4/local128 bf16" if args.protect else "")),
                    "kv_tokens_per_step_per_gpu": tok_per_step, "l2": "flushed (256 MB write) before every timed step",
                    "parallelism": f"replicas x{ws_world} (independent sequences)"},
         "us_per_step": round(ms_step_max * 1e3, 2),
@@ -336,7 +349,7 @@ def run_native(args, ws_world: int, rank: int, local: int):
         "wall_s_timed_loop": round(t_wall, 3),
     }
     if rank == 0 and ws_world == 1 and not args.no_cpu_baseline:
-        res["cpu_baseline"] = cpu_baseline(w, args.bf16_cache, budget_s=15.0)
+        res["cpu_baseline"] = cpu_baseline(w, args.bf16_cache, budget_s=15.0, protect=args.protect)
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
@@ -382,7 +395,8 @@ def run_e2e(state: Workspace, K: int, flush, dev, tokens: float, n_world: int, d
 
 
 # ------------------------------------------------------------------ oracle
-def oracle_step_sample(w: W.Workload, bf16: bool, budget_s: float, max_seqs: int | None = None):
+def oracle_step_sample(w: W.Workload, bf16: bool, budget_s: float, max_seqs: int | None = None,
+                       protect: bool = False):
     """Times the CPU oracle on one decode step (append of the step's tokens,
     read-back and dequantisation of each sequence's cache, fp64 attention) for
     as many sequences as fit in `budget_s`. Returns (tokens, seconds, nseq)."""
@@ -413,6 +427,11 @@ def oracle_step_sample(w: W.Workload, bf16: bool, budget_s: float, max_seqs: int
                                 row[None, :])
             q, s, z = OL.read_sequence(pool, w.c_bits, row, L)
             C, K = OA.dequantize_tokens(q, s, z)
+            if protect:  # sink4/local128 positions attend with their bf16 values
+                from oracle import protection as OP
+                P = OP.protected_positions(L)
+                C, K = np.array(C), np.array(K)
+                C[P], K[P] = lat[P], kp[P]
         OA.attend(ql[b].double().numpy(), qp[b].double().numpy(), C, K, TAU)
         tot_s += time.perf_counter() - t0
         tot_tok += L
@@ -429,8 +448,8 @@ def cpu_cores() -> int:
         return os.cpu_count() or 1
 
 
-def cpu_baseline(w: W.Workload, bf16: bool, budget_s: float):
-    tok, sec, nseq = oracle_step_sample(w, bf16, budget_s)
+def cpu_baseline(w: W.Workload, bf16: bool, budget_s: float, protect: bool = False):
+    tok, sec, nseq = oracle_step_sample(w, bf16, budget_s, protect=protect)
     return {"value": round(tok / sec, 1), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
             "sample": f"{nseq} of {w.batch} sequences of one decode step ({tok} KV tokens, "
                       f"{w.heads} heads): append + cache read-back + dequantisation + fp64 attention, "
@@ -444,7 +463,8 @@ def run_reference(args, ws_world: int, rank: int):
     # Each step is a bounded sample: at most 4 sequences of the step.
     steps = []
     for i in range(args.warmup + args.steps):
-        tok, sec, nseq = oracle_step_sample(w, args.bf16_cache, budget_s=1e9, max_seqs=min(4, w.batch))
+        tok, sec, nseq = oracle_step_sample(w, args.bf16_cache, budget_s=1e9, max_seqs=min(4, w.batch),
+                                            protect=args.protect)
         if i >= args.warmup:
             steps.append((tok, sec))
     tok = sum(t for t, _ in steps)

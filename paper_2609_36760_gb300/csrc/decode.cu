@@ -680,7 +680,9 @@ __device__ bool epilogue(const Params& p, const SegEnd& e, Ctrl& ctl, uint32_t t
   return true;
 }
 
-template <int CB, int HG>
+// PROT: the cache has sink4/local128 protection rows (a separate instantiation,
+// so the unprotected kernel carries none of that code).
+template <int CB, int HG, bool PROT>
 __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ctl, uint32_t tmem, int warp,
                             int lane) {
   using C = Cols<HG>;
@@ -718,7 +720,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     ref0.b = sc.u / p.n_hg;
   }
   // A protected row reads its BF16 row instead of the packed cache.
-  const uint8_t* psrc_cur = prot_row(p, ref0, row);
+  const uint8_t* psrc_cur = PROT ? prot_row(p, ref0, row) : nullptr;
   const uint8_t* blk_cur = psrc_cur != nullptr ? nullptr : resolve_row<CB>(p, ref0, row, valid_cur);
   if constexpr (CB != 16) {
 #pragma unroll
@@ -742,7 +744,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     // The next tile's block pointer (its table entry was loaded a tile ago)
     // and the table entry of the tile after it.
     bool valid_nx = false;
-    const uint8_t* psrc_nx = prot_row(p, ref_nx, row);
+    const uint8_t* psrc_nx = PROT ? prot_row(p, ref_nx, row) : nullptr;
     const uint8_t* blk_nx = psrc_nx != nullptr ? nullptr : resolve_row<CB>(p, ref_nx, row, valid_nx);
     Sched nn = nx;
     nn.next();
@@ -754,13 +756,6 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     for (int kc = 0; kc < kMyChunks; ++kc) {
       const int k = 2 * kc + par;
       if (k >= kNumChunks) break;
-      uint4 pv[CB == 16 ? 1 : 8];  // a protected row's chunk, loaded before the slot wait
-      if constexpr (CB != 16) {
-        if (psrc_cur != nullptr) {
-#pragma unroll
-          for (int i = 0; i < 8; ++i) pv[i] = ldg_nc_v4(psrc_cur + k * 128 + i * 16);
-        }
-      }
       if (!(ok = wwait(slot_bar(ctl, k), (it & 1u) ^ 1u, ctl, kSiteDqSlot, p.dev_err))) break;
       if (lane == 0) QMLA_TRACE(88 + warp, it);  // (overwritten per chunk: last slot wait)
       if constexpr (CB == 16) {
@@ -779,7 +774,10 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
 #pragma unroll
         for (int i = 0; i < 8; ++i) cur[i] = nxt[i];
       } else {
-        if (psrc_cur != nullptr) {
+        if (PROT && psrc_cur != nullptr) {
+          uint4 pv[8];  // the protected row's 64 bf16 values of chunk k
+#pragma unroll
+          for (int i = 0; i < 8; ++i) pv[i] = ldg_nc_v4(psrc_cur + k * 128 + i * 16);
           store_row_prot<CB>(chunks + k * kChunkBytes, row, pv, k);
         } else {
           store_row<CB>(chunks + k * kChunkBytes, row, f[kc], CB == 4 || k == 8);
@@ -1015,7 +1013,7 @@ __device__ void mma_thread(const Params& p, Sched sc, uint32_t chunks, uint8_t* 
   wait_ok(mbar_wait(&ctl.fin, 0, kWaitNs, nullptr), kSiteMmaFin, ctl, p.dev_err);
 }
 
-template <int CB, int HG>
+template <int CB, int HG, bool PROT>
 __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -1060,7 +1058,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   Sched sc;
   sc.init(p.prefix, p.cta_info[blockIdx.x], p.batch * p.n_hg, blockIdx.x, gridDim.x);
   if (warp < kWorkers) {
-    worker_role<CB, HG>(p, sc, chunks, ctl, tmem, warp, lane);
+    worker_role<CB, HG, PROT>(p, sc, chunks, ctl, tmem, warp, lane);
   } else {
     mma_thread<HG>(p, sc, chunks, qsmem, ctl, tmem);
   }
@@ -1228,14 +1226,14 @@ __global__ void __launch_bounds__(128) combine_kernel(const Params p) {
   if (lane == 0 && p.lse != nullptr) p.lse[static_cast<size_t>(b) * p.heads + h0 + h] = (M + log2f(l)) * kLn2;
 }
 
-template <int CB, int HG>
+template <int CB, int HG, bool PROT>
 cudaError_t launch_impl(const Params& prm, cudaStream_t stream, cudaEvent_t ev0, cudaEvent_t ev1) {
   static int configured_device = -1;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (configured_device != dev) {
-    e = cudaFuncSetAttribute(decode_main<CB, HG>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<HG>::kSmem);
+    e = cudaFuncSetAttribute(decode_main<CB, HG, PROT>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<HG>::kSmem);
     if (e != cudaSuccess) return e;
     configured_device = dev;
   }
@@ -1245,18 +1243,18 @@ cudaError_t launch_impl(const Params& prm, cudaStream_t stream, cudaEvent_t ev0,
   prep_kernel<CB, HG><<<prep_blocks, kPrepThreads, 0, stream>>>(prm);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (ev0 != nullptr && (e = cudaEventRecord(ev0, stream)) != cudaSuccess) return e;
-  decode_main<CB, HG><<<prm.grid, kThreads, Cfg<HG>::kSmem, stream>>>(prm);
+  decode_main<CB, HG, PROT><<<prm.grid, kThreads, Cfg<HG>::kSmem, stream>>>(prm);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (ev1 != nullptr && (e = cudaEventRecord(ev1, stream)) != cudaSuccess) return e;
   combine_kernel<HG><<<dim3(static_cast<unsigned>(units), (HG + 3) / 4), 128, 0, stream>>>(prm);
   return cudaGetLastError();
 }
 
-template <int CB>
+template <int CB, bool PROT>
 cudaError_t launch_hg(int hg, const Params& prm, cudaStream_t stream, cudaEvent_t ev0, cudaEvent_t ev1) {
-  if (hg == 16) return launch_impl<CB, 16>(prm, stream, ev0, ev1);
-  if (hg == 32) return launch_impl<CB, 32>(prm, stream, ev0, ev1);
-  return launch_impl<CB, 64>(prm, stream, ev0, ev1);
+  if (hg == 16) return launch_impl<CB, 16, PROT>(prm, stream, ev0, ev1);
+  if (hg == 32) return launch_impl<CB, 32, PROT>(prm, stream, ev0, ev1);
+  return launch_impl<CB, 64, PROT>(prm, stream, ev0, ev1);
 }
 
 }  // namespace
@@ -1316,9 +1314,14 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
 #else
   prm.trace = nullptr;
 #endif
-  if (a.cache_kind == 4) return launch_hg<4>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
-  if (a.cache_kind == 2) return launch_hg<2>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
-  return launch_hg<16>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
+  const bool prot = prm.prot != nullptr;
+  if (a.cache_kind == 4)
+    return prot ? launch_hg<4, true>(hg, prm, stream, a.ev_before_main, a.ev_after_main)
+                : launch_hg<4, false>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
+  if (a.cache_kind == 2)
+    return prot ? launch_hg<2, true>(hg, prm, stream, a.ev_before_main, a.ev_after_main)
+                : launch_hg<2, false>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
+  return launch_hg<16, false>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
 }
 
 #ifdef QMLA_TRACE_BUILD
