@@ -721,6 +721,12 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
   }
   // A protected row reads its BF16 row instead of the packed cache.
   const uint8_t* psrc_cur = PROT ? prot_row(p, ref0, row) : nullptr;
+  if constexpr (PROT) {
+    if (psrc_cur != nullptr) {
+#pragma unroll
+      for (int i = 0; i < kDqk * 2 / 128; ++i) asm volatile("prefetch.global.L2 [%0];" ::"l"(psrc_cur + i * 128));
+    }
+  }
   const uint8_t* blk_cur = psrc_cur != nullptr ? nullptr : resolve_row<CB>(p, ref0, row, valid_cur);
   if constexpr (CB != 16) {
 #pragma unroll
@@ -745,6 +751,14 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     // and the table entry of the tile after it.
     bool valid_nx = false;
     const uint8_t* psrc_nx = PROT ? prot_row(p, ref_nx, row) : nullptr;
+    if constexpr (PROT) {
+      // The next tile's protected rows into L2 now (no registers held): their
+      // chunk loads come after each slot wait and would otherwise miss to DRAM.
+      if (psrc_nx != nullptr) {
+#pragma unroll
+        for (int i = 0; i < kDqk * 2 / 128; ++i) asm volatile("prefetch.global.L2 [%0];" ::"l"(psrc_nx + i * 128));
+      }
+    }
     const uint8_t* blk_nx = psrc_nx != nullptr ? nullptr : resolve_row<CB>(p, ref_nx, row, valid_nx);
     Sched nn = nx;
     nn.next();
@@ -777,7 +791,9 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
         if (PROT && psrc_cur != nullptr) {
           uint4 pv[8];  // the protected row's 64 bf16 values of chunk k
 #pragma unroll
-          for (int i = 0; i < 8; ++i) pv[i] = ldg_nc_v4(psrc_cur + k * 128 + i * 16);
+          // L1-allocating loads: the eight 16-byte pieces of the row's 128-byte
+          // line come from one L1 fill instead of eight L2 reads.
+          for (int i = 0; i < 8; ++i) pv[i] = __ldg(reinterpret_cast<const uint4*>(psrc_cur + k * 128) + i);
           store_row_prot<CB>(chunks + k * kChunkBytes, row, pv, k);
         } else {
           store_row<CB>(chunks + k * kChunkBytes, row, f[kc], CB == 4 || k == 8);
