@@ -16,8 +16,11 @@ storage    the persistent-storage closed form (App. C.5, Eq. physical_cache_stor
 protection sink4/local128 BF16 protection: the protected set, this library's
            protection-buffer rows and writer rule, protected attention (App. C.5,
            "BF16 protection and cache lifecycle")
+paper_format the paper's own 20,480-byte page: bf16 content scales, fp32 RoPE
+           scale, uint8 zero points, its quantiser staging, writer and reader
+           (App. C.4, App. C.5 storage layout)
 
 Every function is pinned by tests under ``tests/test_oracle_*.py``; nothing in
 this package is marked "parity unpinned".
 """
-from . import attention, layout, protection, quantizer, storage  # noqa: F401
+from . import attention, layout, paper_format, protection, quantizer, storage  # noqa: F401
