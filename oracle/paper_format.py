@@ -1,7 +1,7 @@
-"""The paper's own C4R4 page format, in fp64 (App. C.4, "Native execution stores
-content scales in BF16 and RoPE scales in FP32 and dequantizes using the stored
-scales"; App. C.5, storage layout: 20,480 bytes per 64-token page, 320 bytes per
-token). Test infrastructure: used by tests/ only.
+"""The paper's own C4R4 page format, in fp64. App. C.4: the native kernels keep
+each content group's scale as bf16 and the RoPE group's scale as fp32, and
+dequantise with those stored values. App. C.5, storage layout: 20,480 bytes per
+64-token page, 320 bytes per token. Test infrastructure: used by tests/ only.
 
 Quantiser (App. C.4: s = max(x_max - x_min, 1e-8) / m, z = clip(rne(-x_min / s), 0, m),
 q = clip(rne(x / s + z), 0, m), x_hat = s (q - z), m = 15 for 4-bit groups), with the
