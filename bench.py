@@ -49,6 +49,8 @@ def parse():
     ap.add_argument("--bf16-cache", action="store_true", help="decode the BF16 comparison cache instead")
     ap.add_argument("--protect", action="store_true",
                     help="sink4/local128 BF16 protection (the paper's C4R4 serving configuration)")
+    ap.add_argument("--c4r4", action="store_true",
+                    help="store the INT4 cache in the paper's own 20,480-byte page (bf16/fp32 scales, uint8 zeros)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
@@ -70,11 +72,11 @@ def load_peaks():
     return dict(FALLBACK_PEAKS), "fallback"
 
 
-def workload_cost(w: W.Workload, lens: list[int], bf16: bool):
+def workload_cost(w: W.Workload, lens: list[int], bf16: bool, c4r4: bool = False):
     """Algorithmic FLOPs and HBM bytes of one decode launch (see the design notes)."""
     tokens = sum(lens)
     flops = 2.0 * w.heads * (576 + 512) * tokens
-    per_tok = 1152 if bf16 else (324 if w.c_bits == 4 else 196)
+    per_tok = 1152 if bf16 else (320 if c4r4 else (324 if w.c_bits == 4 else 196))
     nbytes = tokens * per_tok + w.batch * w.heads * (576 * 2 + 512 * 4 + 4)
     return flops, nbytes
 
@@ -156,15 +158,19 @@ def decode_cu_hash() -> str:
 class Workspace:
     """GPU state of one workload: pool, block table, per-step inputs."""
 
-    def __init__(self, w: W.Workload, bf16: bool, dev: torch.device, nsteps: int, protect: bool = False):
+    def __init__(self, w: W.Workload, bf16: bool, dev: torch.device, nsteps: int, protect: bool = False,
+                 c4r4: bool = False):
         import paper_2609_36760_gb300 as Q
         self.Q = Q
         self.w, self.bf16, self.dev = w, bf16, dev
         self.protect = protect and not bf16
+        self.c4r4 = c4r4 and not bf16
+        if self.c4r4 and w.c_bits != 4:
+            raise SystemExit("--c4r4 stores INT4 content: pick a workload with c_bits = 4")
         self.prefill = W.seq_lengths(w)
         table, nblocks = W.block_table(w)
         self.table = table.to(dev)
-        bb = Q.bf16_block_bytes() if bf16 else Q.block_bytes(w.c_bits)
+        bb = Q.bf16_block_bytes() if bf16 else (Q.c4r4_page_bytes() if self.c4r4 else Q.block_bytes(w.c_bits))
         self.pool = torch.zeros((nblocks, bb), dtype=torch.uint8, device=dev)
         self.err = torch.zeros(1, dtype=torch.int32, device=dev)
         # per-request 132 x 576 bf16 protection rows (152,064 bytes each)
@@ -209,7 +215,10 @@ class Workspace:
     def _append(self, lat, kp, sid, pos, lens_after=None):
         if lat.shape[0] == 0:
             return
-        if self.protect:
+        if self.c4r4:
+            self.Q.quant_append_c4r4(self.pool, lat, kp, sid, pos, self.table, self.err,
+                                     seq_lens=lens_after if self.protect else None, prot=self.prot)
+        elif self.protect:
             self.Q.quant_append_protected(self.pool, self.w.c_bits, lat, kp, sid, pos, self.table, lens_after,
                                           self.prot, self.err)
         elif self.bf16:
@@ -222,7 +231,10 @@ class Workspace:
         out = self.out if out is None else out
         lse = self.lse if lse is None else lse
         self._append(d["lat"], d["kp"], d["sid"], d["pos"], d["lens"])
-        if self.protect:
+        if self.c4r4:
+            self.Q.mla_decode_c4r4(self.pool, d["ql"], d["qp"], self.table, d["lens"], TAU, out, lse, self.ws,
+                                   self.err, prot=self.prot)
+        elif self.protect:
             self.Q.mla_decode_protected(self.pool, self.w.c_bits, d["ql"], d["qp"], self.table, d["lens"], self.prot,
                                         TAU, out, lse, self.ws, self.err)
         elif self.bf16:
@@ -247,7 +259,7 @@ def run_native(args, ws_world: int, rank: int, local: int):
         dist.init_process_group("nccl", device_id=dev)
     w = W.WORKLOADS[args.workload]
     K, Wm = args.steps, args.warmup
-    state = Workspace(w, args.bf16_cache, dev, K + Wm, protect=args.protect)
+    state = Workspace(w, args.bf16_cache, dev, K + Wm, protect=args.protect, c4r4=args.c4r4)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # larger than the 126 MB L2
     stream = torch.cuda.current_stream(dev)
 
@@ -306,7 +318,7 @@ def run_native(args, ws_world: int, rank: int, local: int):
 
     # roofline of the main decode kernel
     peaks, peak_src = load_peaks()
-    flops, nbytes = workload_cost(w, lens_all[0], args.bf16_cache)
+    flops, nbytes = workload_cost(w, lens_all[0], args.bf16_cache, state.c4r4)
     t_tc = flops / (peaks["bf16_tflops"] * 1e12)
     t_hbm = nbytes / (peaks["hbm_gbs"] * 1e9)
     tensor_bound = t_tc >= t_hbm
@@ -320,7 +332,9 @@ def run_native(args, ws_world: int, rank: int, local: int):
     roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
     prof = profile_traffic(decode_cu_hash())
     roof["traffic"] = (prof["dram_bytes_per_launch"] if prof and prof.get("workload") == args.workload
-                       and bool(prof.get("bf16_cache")) == bool(args.bf16_cache) else None)
+                       and bool(prof.get("bf16_cache")) == bool(args.bf16_cache)
+                       and bool(prof.get("protect")) == bool(args.protect)
+                       and bool(prof.get("c4r4")) == bool(state.c4r4) else None)
     roof["kernel"] = "decode_main"
     roof["kernel_us"] = round(ms_main * 1e3, 2)
     roof["algorithmic_flops"] = flops
@@ -337,8 +351,7 @@ def run_native(args, ws_world: int, rank: int, local: int):
         "ms_per_step": round(ms_step_max, 5), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "f16", "data": "synthetic (seeded generators, workloads/synthetic.py)",
         "config": {"workload": w.name, "batch_per_gpu": w.batch, "heads": w.heads, "c_bits": w.c_bits,
-                   "pe_bits": 4, "cache": "bf16" if args.bf16_cache else (
-                       f"int{w.c_bits}/int4 packed" + (" + sink4/local128 bf16" if args.protect else "")),
+                   "pe_bits": 4, "cache": cache_name(w, args.bf16_cache, args.protect, state.c4r4),
                    "kv_tokens_per_step_per_gpu": tok_per_step, "l2": "flushed (256 MB write) before every timed step",
                    "parallelism": f"replicas x{ws_world} (independent sequences)"},
         "us_per_step": round(ms_step_max * 1e3, 2),
@@ -349,12 +362,20 @@ def run_native(args, ws_world: int, rank: int, local: int):
         "wall_s_timed_loop": round(t_wall, 3),
     }
     if rank == 0 and ws_world == 1 and not args.no_cpu_baseline:
-        res["cpu_baseline"] = cpu_baseline(w, args.bf16_cache, budget_s=15.0, protect=args.protect)
+        res["cpu_baseline"] = cpu_baseline(w, args.bf16_cache, budget_s=15.0, protect=args.protect,
+                                           c4r4=state.c4r4)
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
     if rank == 0:
         print(json.dumps(res), flush=True)
+
+
+def cache_name(w: W.Workload, bf16: bool, protect: bool, c4r4: bool) -> str:
+    if bf16:
+        return "bf16"
+    base = "c4r4 paper page (bf16 content / fp32 rope scales, uint8 zeros)" if c4r4 else f"int{w.c_bits}/int4 packed"
+    return base + (" + sink4/local128 bf16" if protect else "")
 
 
 def run_e2e(state: Workspace, K: int, flush, dev, tokens: float, n_world: int, dist):
@@ -396,13 +417,14 @@ def run_e2e(state: Workspace, K: int, flush, dev, tokens: float, n_world: int, d
 
 # ------------------------------------------------------------------ oracle
 def oracle_step_sample(w: W.Workload, bf16: bool, budget_s: float, max_seqs: int | None = None,
-                       protect: bool = False):
+                       protect: bool = False, c4r4: bool = False):
     """Times the CPU oracle on one decode step (append of the step's tokens,
     read-back and dequantisation of each sequence's cache, fp64 attention) for
     as many sequences as fit in `budget_s`. Returns (tokens, seconds, nseq)."""
     import numpy as np
     from oracle import attention as OA
     from oracle import layout as OL
+    from oracle import paper_format as OF
 
     prefill = W.seq_lengths(w)
     gains = W.channel_gains(w)
@@ -415,23 +437,31 @@ def oracle_step_sample(w: W.Workload, bf16: bool, budget_s: float, max_seqs: int
         lat = W.latent_for_seq(w, b, L, gains).double().numpy()
         kp = W.kpe_for_seq(w, b, L).double().numpy()
         row = np.arange((L + 63) // 64, dtype=np.int64)
-        if not bf16:
+        if c4r4:
+            pool = np.zeros((len(row), OF.PAGE_BYTES), np.uint8)
+            OF.write_tokens(pool, lat[:n], kp[:n], np.zeros(n, np.int64), np.arange(n), row[None, :])
+        elif not bf16:
             pool = np.zeros((len(row), OL.block_bytes(w.c_bits)), np.uint8)
             OL.write_tokens(pool, w.c_bits, lat[:n], kp[:n], np.zeros(n, np.int64), np.arange(n), row[None, :])
         t0 = time.perf_counter()
         if bf16:
             C, K = lat, kp
+        elif c4r4:
+            if w.append:
+                OF.write_tokens(pool, lat[n:L], kp[n:L], np.zeros(L - n, np.int64), np.arange(n, L), row[None, :])
+            q, s, z = OF.read_sequence(pool, row, L)
+            C, K = OF.dequantize_tokens(q, s, z)
         else:
             if w.append:
                 OL.write_tokens(pool, w.c_bits, lat[n:L], kp[n:L], np.zeros(L - n, np.int64), np.arange(n, L),
                                 row[None, :])
             q, s, z = OL.read_sequence(pool, w.c_bits, row, L)
             C, K = OA.dequantize_tokens(q, s, z)
-            if protect:  # sink4/local128 positions attend with their bf16 values
-                from oracle import protection as OP
-                P = OP.protected_positions(L)
-                C, K = np.array(C), np.array(K)
-                C[P], K[P] = lat[P], kp[P]
+        if protect and not bf16:  # sink4/local128 positions attend with their bf16 values
+            from oracle import protection as OP
+            P = OP.protected_positions(L)
+            C, K = np.array(C), np.array(K)
+            C[P], K[P] = lat[P], kp[P]
         OA.attend(ql[b].double().numpy(), qp[b].double().numpy(), C, K, TAU)
         tot_s += time.perf_counter() - t0
         tot_tok += L
@@ -448,8 +478,8 @@ def cpu_cores() -> int:
         return os.cpu_count() or 1
 
 
-def cpu_baseline(w: W.Workload, bf16: bool, budget_s: float, protect: bool = False):
-    tok, sec, nseq = oracle_step_sample(w, bf16, budget_s, protect=protect)
+def cpu_baseline(w: W.Workload, bf16: bool, budget_s: float, protect: bool = False, c4r4: bool = False):
+    tok, sec, nseq = oracle_step_sample(w, bf16, budget_s, protect=protect, c4r4=c4r4)
     return {"value": round(tok / sec, 1), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
             "sample": f"{nseq} of {w.batch} sequences of one decode step ({tok} KV tokens, "
                       f"{w.heads} heads): append + cache read-back + dequantisation + fp64 attention, "
@@ -464,7 +494,7 @@ def run_reference(args, ws_world: int, rank: int):
     steps = []
     for i in range(args.warmup + args.steps):
         tok, sec, nseq = oracle_step_sample(w, args.bf16_cache, budget_s=1e9, max_seqs=min(4, w.batch),
-                                            protect=args.protect)
+                                            protect=args.protect, c4r4=args.c4r4 and not args.bf16_cache)
         if i >= args.warmup:
             steps.append((tok, sec))
     tok = sum(t for t, _ in steps)
@@ -475,7 +505,8 @@ def run_reference(args, ws_world: int, rank: int):
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
            "data": "synthetic (seeded generators, workloads/synthetic.py)",
            "config": {"workload": w.name, "batch_per_gpu": w.batch, "heads": w.heads, "c_bits": w.c_bits,
-                      "pe_bits": 4, "sample_per_step": f"{min(4, w.batch)} sequences"},
+                      "pe_bits": 4, "cache": cache_name(w, args.bf16_cache, args.protect, args.c4r4),
+                      "sample_per_step": f"{min(4, w.batch)} sequences"},
            "cpu_baseline": {"value": round(value, 1), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                             "sample": f"{min(4, w.batch)} of {w.batch} sequences per step, {len(steps)} steps"},
            "e2e": {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}

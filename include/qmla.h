@@ -13,6 +13,8 @@
  *   qmla_mla_decode     split-KV decode attention over the packed cache, plus the
  *                       split-result combination (Eq. mla_compact; App. C.5
  *                       "global attention normalization")
+ *   *_protected         the same with sink4/local128 BF16 protection (App. C.5)
+ *   *_c4r4              the same over the paper's own 20,480-byte INT4 page
  *
  * Conventions for every call
  * --------------------------
@@ -201,6 +203,50 @@ int qmla_mla_decode_bf16cache(const void* pool_dev, int num_blocks, const uint16
                               const int32_t* seq_lens_dev, float softmax_scale, float* out_dev,
                               float* lse_dev, void* workspace_dev, size_t workspace_bytes,
                               uint32_t* dev_err_dev, qmla_stream_t stream);
+
+/*
+ * The paper's own INT4 page ("C4R4": 4-bit content, 4-bit RoPE key; App. C.5,
+ * storage layout; App. C.4, scale precisions). Same codes, groups and packing as
+ * the c_bits = 4 block above; the metadata differ: per token and group a bf16
+ * scale for content groups, an fp32 scale for the RoPE group, and a uint8 zero
+ * point. Staging (App. C.4 with m = 15; d = RN_f32(x_max - x_min)):
+ *     content  s = RN_bf16(RN_f32(max(d, 1e-8) / 15))
+ *     RoPE     s = RN_f32(max(d, 1e-8) / 15)
+ *     z = clip(rne(RN_f32(-x_min / s)), 0, 15);  q = clip(rne(RN_f32(RN_f32(x / s) + z)), 0, 15)
+ * (for content groups the fp32 quotients give the exact-arithmetic codes, since
+ * a bf16 x over a bf16 s is never within fp32 rounding of a half-integer).
+ * A page of 64 token slots, 20480 bytes (320 per token):
+ *     [0, 16384)       content codes   [group 8][slot 64][32 bytes]
+ *     [16384, 18432)   RoPE-key codes  [slot 64][32 bytes]
+ *     [18432, 19456)   content scales  [group 8][slot 64] bf16
+ *     [19456, 19712)   RoPE scales     [slot 64] fp32
+ *     [19712, 20288)   zero points     [group 9][slot 64] uint8 (group 8: RoPE key)
+ *     [20288, 20480)   padding, never written or read
+ * The decode's fp16 tile value of a code is RN_f16(s (q - z)) for content and
+ * RN_f16(RN_f32(s (q - z))) for the RoPE key.
+ */
+size_t qmla_c4r4_page_bytes(void);
+
+/* qmla_quant_append into pages of the paper's format (qmla_c4r4_page_bytes()
+ * bytes each). prot_dev is optional: NULL writes the packed pages only; non-NULL
+ * also writes the sink4/local128 protection rows as qmla_quant_append_protected
+ * does, and then seq_lens_dev (lengths after this call) must be non-NULL and
+ * latent_dev, k_pe_dev, prot_dev 16-byte aligned. Errors as qmla_quant_append. */
+int qmla_quant_append_c4r4(void* pool_dev, int num_blocks, const uint16_t* latent_dev, const uint16_t* k_pe_dev,
+                           const int32_t* seq_ids_dev, const int32_t* positions_dev, int n,
+                           const int32_t* block_table_dev, int num_seqs, int max_blocks,
+                           const int32_t* seq_lens_dev, void* prot_dev, uint32_t* dev_err_dev,
+                           qmla_stream_t stream);
+
+/* qmla_mla_decode over pages of the paper's format. prot_dev NULL attends over
+ * the packed pages only; non-NULL (16-byte aligned) applies sink4/local128
+ * protection as qmla_mla_decode_protected does. Outputs, workspace
+ * (qmla_decode_workspace_bytes) and errors as qmla_mla_decode. */
+int qmla_mla_decode_c4r4(const void* pool_dev, int num_blocks, const uint16_t* q_latent_dev,
+                         const uint16_t* q_pe_dev, int batch, int heads, const int32_t* block_table_dev,
+                         int max_blocks, const int32_t* seq_lens_dev, const void* prot_dev, float softmax_scale,
+                         float* out_dev, float* lse_dev, void* workspace_dev, size_t workspace_bytes,
+                         uint32_t* dev_err_dev, qmla_stream_t stream);
 
 /* Measurement hook. While set (per host thread), every qmla_mla_decode* call
  * records the caller-owned CUDA events `before_main` and `after_main`

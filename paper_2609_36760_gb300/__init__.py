@@ -73,6 +73,11 @@ def lib():
     L.qmla_mla_decode_protected.argtypes = [vp, i32, i32, vp, vp, i32, i32, vp, i32, vp, vp, f32, vp, vp, vp, sz,
                                             vp, vp]
     L.qmla_mla_decode_protected.restype = i32
+    L.qmla_c4r4_page_bytes.argtypes, L.qmla_c4r4_page_bytes.restype = [], sz
+    L.qmla_quant_append_c4r4.argtypes = [vp, i32, vp, vp, vp, vp, i32, vp, i32, i32, vp, vp, vp, vp]
+    L.qmla_quant_append_c4r4.restype = i32
+    L.qmla_mla_decode_c4r4.argtypes = [vp, i32, vp, vp, i32, i32, vp, i32, vp, vp, f32, vp, vp, vp, sz, vp, vp]
+    L.qmla_mla_decode_c4r4.restype = i32
     _lib = L
     return L
 
@@ -174,6 +179,38 @@ def mla_decode_protected(pool: torch.Tensor, c_bits: int, q_latent: torch.Tensor
                                          workspace.numel() * workspace.element_size(), _ptr(dev_err),
                                          _stream(stream))
     _check("qmla_mla_decode_protected", st)
+
+
+def c4r4_page_bytes() -> int:
+    """Bytes of one 64-token page of the paper's INT4 format (20480)."""
+    return int(lib().qmla_c4r4_page_bytes())
+
+
+def quant_append_c4r4(pool: torch.Tensor, latent: torch.Tensor, k_pe: torch.Tensor, seq_ids: torch.Tensor | None,
+                      positions: torch.Tensor, block_table: torch.Tensor, dev_err: torch.Tensor,
+                      seq_lens: torch.Tensor | None = None, prot: torch.Tensor | None = None, stream=None) -> None:
+    """qmla_quant_append_c4r4: pages of the paper's format; with prot (and
+    seq_lens = lengths after this call) also the sink/recent bf16 rows."""
+    n = latent.shape[0]
+    st = lib().qmla_quant_append_c4r4(_ptr(pool), pool.shape[0], _ptr(latent), _ptr(k_pe), _ptr(seq_ids),
+                                      _ptr(positions), n, _ptr(block_table), block_table.shape[0],
+                                      block_table.shape[1], _ptr(seq_lens), _ptr(prot), _ptr(dev_err),
+                                      _stream(stream))
+    _check("qmla_quant_append_c4r4", st)
+
+
+def mla_decode_c4r4(pool: torch.Tensor, q_latent: torch.Tensor, q_pe: torch.Tensor, block_table: torch.Tensor,
+                    seq_lens: torch.Tensor, softmax_scale: float, out: torch.Tensor, lse: torch.Tensor | None,
+                    workspace: torch.Tensor, dev_err: torch.Tensor, prot: torch.Tensor | None = None,
+                    stream=None) -> None:
+    """qmla_mla_decode_c4r4: mla_decode over pages of the paper's format, with
+    sink4/local128 protection when prot [B, 132, 576] is given."""
+    B, H = q_latent.shape[0], q_latent.shape[1]
+    st = lib().qmla_mla_decode_c4r4(_ptr(pool), pool.shape[0], _ptr(q_latent), _ptr(q_pe), B, H, _ptr(block_table),
+                                    block_table.shape[1], _ptr(seq_lens), _ptr(prot), float(softmax_scale),
+                                    _ptr(out), _ptr(lse), _ptr(workspace),
+                                    workspace.numel() * workspace.element_size(), _ptr(dev_err), _stream(stream))
+    _check("qmla_mla_decode_c4r4", st)
 
 
 def mla_decode_bf16cache(pool: torch.Tensor, q_latent: torch.Tensor, q_pe: torch.Tensor, block_table: torch.Tensor,

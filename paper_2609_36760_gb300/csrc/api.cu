@@ -203,6 +203,40 @@ int qmla_mla_decode_protected(const void* pool_dev, int c_bits, int num_blocks, 
                        dev_err_dev, stream, prot_dev);
 }
 
+size_t qmla_c4r4_page_bytes(void) { return qmla::BlockLayout<qmla::kC4R4>::kBytes; }
+
+int qmla_quant_append_c4r4(void* pool_dev, int num_blocks, const uint16_t* latent_dev, const uint16_t* k_pe_dev,
+                           const int32_t* seq_ids_dev, const int32_t* positions_dev, int n,
+                           const int32_t* block_table_dev, int num_seqs, int max_blocks,
+                           const int32_t* seq_lens_dev, void* prot_dev, uint32_t* dev_err_dev,
+                           qmla_stream_t stream) {
+  int st = append_common_checks(pool_dev, num_blocks, latent_dev, k_pe_dev, positions_dev, n, block_table_dev,
+                                num_seqs, max_blocks);
+  if (st != QMLA_OK) return st;
+  if (prot_dev != nullptr &&
+      (seq_lens_dev == nullptr || !aligned(prot_dev, 16) || !aligned(seq_lens_dev, 4) ||
+       !aligned(latent_dev, 16) || !aligned(k_pe_dev, 16)))
+    return QMLA_ERR_INVALID_ARG;
+  if (n == 0) return QMLA_OK;
+  DevInfo di;
+  if ((st = current_device_info(di)) != QMLA_OK) return st;
+  cudaError_t e = qmla::launch_quant_append(pool_dev, qmla::kC4R4, num_blocks, latent_dev, k_pe_dev, seq_ids_dev,
+                                            positions_dev, n, block_table_dev, num_seqs, max_blocks,
+                                            dev_err_dev, reinterpret_cast<cudaStream_t>(stream), prot_dev,
+                                            prot_dev != nullptr ? seq_lens_dev : nullptr);
+  return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
+}
+
+int qmla_mla_decode_c4r4(const void* pool_dev, int num_blocks, const uint16_t* q_latent_dev,
+                         const uint16_t* q_pe_dev, int batch, int heads, const int32_t* block_table_dev,
+                         int max_blocks, const int32_t* seq_lens_dev, const void* prot_dev, float softmax_scale,
+                         float* out_dev, float* lse_dev, void* workspace_dev, size_t workspace_bytes,
+                         uint32_t* dev_err_dev, qmla_stream_t stream) {
+  return decode_common(pool_dev, qmla::kC4R4, num_blocks, q_latent_dev, q_pe_dev, batch, heads, block_table_dev,
+                       max_blocks, seq_lens_dev, softmax_scale, out_dev, lse_dev, workspace_dev, workspace_bytes,
+                       dev_err_dev, stream, prot_dev);
+}
+
 int qmla_mla_decode_bf16cache(const void* pool_dev, int num_blocks, const uint16_t* q_latent_dev,
                               const uint16_t* q_pe_dev, int batch, int heads, const int32_t* block_table_dev,
                               int max_blocks, const int32_t* seq_lens_dev, float softmax_scale, float* out_dev,

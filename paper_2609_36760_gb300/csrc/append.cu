@@ -1,6 +1,7 @@
 // Quantise-and-pack cache writer (App. C.4 quantiser; App. C.5 cache update:
 // content- and RoPE-cache quantisation, integer packing and slot-mapped page
-// insertion), and the plain BF16 writer for the comparison cache.
+// insertion) for this library's block and for the paper's own page, and the
+// plain BF16 writer for the comparison cache.
 //
 // One warp per token. For each of the 9 groups of 64 coordinates, lane l holds
 // coordinates 2l and 2l+1; the group extrema come from warp reductions, every
@@ -35,6 +36,17 @@ __device__ __forceinline__ void group_scale(float xmin, float xmax, int m, float
   if (s == 0.0f) s = 5.9604644775390625e-08f;  // 2^-24, the smallest fp16 subnormal
   if (isinf(s)) s = 65504.0f;
   z = fminf(fmaxf(rintf(__fdiv_rn(-xmin, s)), 0.0f), static_cast<float>(m));
+}
+
+// Scales of the paper's page (App. C.4 with that format's staging): content
+// s = RN_bf16(RN_f32(max(d, 1e-8) / 15)), RoPE s = RN_f32(max(d, 1e-8) / 15);
+// z = clip(rne(-x_min / s), 0, 15) from an fp32 quotient. A bf16 scale and a
+// bf16 input carry 8 significant bits each, so the fp32 quotients of the
+// content path round to the same codes as exact arithmetic would.
+__device__ __forceinline__ void paper_scale(float xmin, float xmax, bool content, float& s, float& z) {
+  const float s32 = __fdiv_rn(fmaxf(xmax - xmin, 1e-8f), 15.0f);
+  s = content ? __bfloat162float(__float2bfloat16_rn(s32)) : s32;
+  z = fminf(fmaxf(rintf(__fdiv_rn(-xmin, s)), 0.0f), 15.0f);
 }
 
 __device__ __forceinline__ uint32_t quant_code(float x, float s, float z, int m) {
@@ -93,6 +105,7 @@ __device__ __forceinline__ void protect_row(uint4* prot, const uint4* latent, co
 
 // prot / lens: the protection buffer [num_seqs][132][576] bf16 and the
 // requests' lengths after this write, or null for an unprotected cache.
+// CB: content bits (4, 2) or kC4R4 for the paper's page (INT4 codes).
 template <int CB>
 __global__ void __launch_bounds__(256) quant_append_kernel(
     uint8_t* __restrict__ pool, int num_blocks, const __nv_bfloat162* __restrict__ latent,
@@ -115,7 +128,7 @@ __global__ void __launch_bounds__(256) quant_append_kernel(
 
 #pragma unroll 1
   for (int g = 0; g < kGroups; ++g) {
-    const int bits = g < 8 ? CB : kPeBits;
+    const int bits = g < 8 ? (CB == kC4R4 ? 4 : CB) : kPeBits;
     const int m = (1 << bits) - 1;
     const __nv_bfloat162 v = g < 8 ? latent[static_cast<size_t>(tok) * (kDc / 2) + g * 32 + lane]
                                    : k_pe[static_cast<size_t>(tok) * (kDr / 2) + lane];
@@ -123,7 +136,11 @@ __global__ void __launch_bounds__(256) quant_append_kernel(
     const float xmin = warp_min_f32(fminf(x0, x1));
     const float xmax = warp_max_f32(fmaxf(x0, x1));
     float s, z;
-    group_scale(xmin, xmax, m, s, z);
+    if constexpr (CB == kC4R4) {
+      paper_scale(xmin, xmax, g < 8, s, z);
+    } else {
+      group_scale(xmin, xmax, m, s, z);
+    }
     const uint32_t code = quant_code(x0, s, z, m) | (quant_code(x1, s, z, m) << bits);
     // Lane l's 2*bits bits sit at bit offset 2*bits*l of the group's code string.
     const int lane_bits = 2 * bits;
@@ -134,8 +151,17 @@ __global__ void __launch_bounds__(256) quant_append_kernel(
       reinterpret_cast<uint32_t*>(blk + L::code_off(g, slot))[lane / lanes_per_word] = word;
     }
     if (lane == 0) {
-      *reinterpret_cast<__half2*>(blk + L::sz_off(g, slot)) =
-          __halves2half2(__float2half_rn(s), __float2half_rn(z));
+      if constexpr (CB == kC4R4) {
+        if (g < 8) {
+          *reinterpret_cast<__nv_bfloat16*>(blk + L::c_scale_off(g, slot)) = __float2bfloat16_rn(s);  // exact
+        } else {
+          *reinterpret_cast<float*>(blk + L::pe_scale_off(slot)) = s;
+        }
+        blk[L::zero_off(g, slot)] = static_cast<uint8_t>(z);
+      } else {
+        *reinterpret_cast<__half2*>(blk + L::sz_off(g, slot)) =
+            __halves2half2(__float2half_rn(s), __float2half_rn(z));
+      }
     }
   }
 }
@@ -169,7 +195,11 @@ cudaError_t launch_quant_append(void* pool, int c_bits, int num_blocks, const ui
   const dim3 grid(static_cast<unsigned>((static_cast<long long>(n) * 32 + 255) / 256));
   auto* lat = reinterpret_cast<const __nv_bfloat162*>(latent);
   auto* kp = reinterpret_cast<const __nv_bfloat162*>(k_pe);
-  if (c_bits == 4) {
+  if (c_bits == kC4R4) {
+    quant_append_kernel<kC4R4><<<grid, block, 0, stream>>>(static_cast<uint8_t*>(pool), num_blocks, lat,
+                                                           kp, seq_ids, positions, n, table, num_seqs,
+                                                           max_blocks, dev_err, static_cast<uint4*>(prot), lens);
+  } else if (c_bits == 4) {
     quant_append_kernel<4><<<grid, block, 0, stream>>>(static_cast<uint8_t*>(pool), num_blocks, lat,
                                                        kp, seq_ids, positions, n, table, num_seqs,
                                                        max_blocks, dev_err, static_cast<uint4*>(prot), lens);

@@ -152,7 +152,7 @@ struct Perm {
   // position p of a piece holds channel at(p): INT4 swaps bits 0 and 1 of p
   // ([0,2,1,3,4,6,5,7]); INT2 rotates them ([0,4,1,5,2,6,3,7]); BF16 keeps p.
   __host__ __device__ static constexpr int at(int p) {
-    if constexpr (CB == 4) {
+    if constexpr (CB == 4 || CB == kC4R4) {
       return (p & 4) | ((p & 1) << 1) | ((p >> 1) & 1);
     } else if constexpr (CB == 2) {
       return ((p & 1) << 2) | (p >> 1);
@@ -175,6 +175,16 @@ __device__ __forceinline__ uint4 ldg_nc_v4(const void* ptr) {
 __device__ __forceinline__ uint32_t ldg_nc_u32(const void* ptr) {
   uint32_t r;
   asm volatile("ld.global.nc.L1::no_allocate.u32 %0, [%1];" : "=r"(r) : "l"(ptr));
+  return r;
+}
+__device__ __forceinline__ uint32_t ldg_nc_u16(const void* ptr) {
+  uint16_t r;
+  asm volatile("ld.global.nc.L1::no_allocate.u16 %0, [%1];" : "=h"(r) : "l"(ptr));
+  return r;
+}
+__device__ __forceinline__ uint32_t ldg_nc_u8(const void* ptr) {
+  uint32_t r;
+  asm volatile("ld.global.nc.L1::no_allocate.u8 %0, [%1];" : "=r"(r) : "l"(ptr));
   return r;
 }
 __device__ __forceinline__ void sts_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
@@ -301,7 +311,8 @@ __device__ __forceinline__ TileInfo tile_info(const Sched& s, const Params& p) {
 // Packed data of one token row for one chunk, fetched ahead of use.
 struct Fetch {
   uint4 a, b;
-  uint32_t sz;
+  uint32_t sz;  // fp16 (s, z) pair; for the paper's page the scale as fp32 bits
+  uint32_t z;   // the paper's page: the uint8 zero point
   bool ok;
 };
 
@@ -369,12 +380,19 @@ __device__ __forceinline__ Fetch fetch_chunk(const uint8_t* blk, bool valid, int
   f.a = make_uint4(0, 0, 0, 0);
   f.b = f.a;
   f.sz = 0;
+  f.z = 0;
   if (!valid) return f;
   using L = BlockLayout<CB>;
   const uint8_t* c = blk + L::code_off(k, slot);
   f.a = ldg_nc_v4(c);
-  if (CB == 4 || k == 8) f.b = ldg_nc_v4(c + 16);
-  f.sz = ldg_nc_u32(blk + L::sz_off(k, slot));
+  if (CB == 4 || CB == kC4R4 || k == 8) f.b = ldg_nc_v4(c + 16);
+  if constexpr (CB == kC4R4) {
+    // bf16 content scale -> fp32 bits by a 16-bit shift; the RoPE scale is fp32
+    f.sz = k < 8 ? ldg_nc_u16(blk + L::c_scale_off(k, slot)) << 16 : ldg_nc_u32(blk + L::pe_scale_off(slot));
+    f.z = ldg_nc_u8(blk + L::zero_off(k, slot));
+  } else {
+    f.sz = ldg_nc_u32(blk + L::sz_off(k, slot));
+  }
   return f;
 }
 
@@ -418,6 +436,66 @@ __device__ __forceinline__ void store_row(uint32_t chunk_base, int row, const Fe
       sts_v4(chunk_base + swz_off(row, 2 * i + 1, 128), dq2(__byte_perm(c0, K, 0x4342), zz, ss),
              dq2(__byte_perm(c1, K, 0x4342), zz, ss), dq2(__byte_perm(c2, K, 0x4342), zz, ss),
              dq2(__byte_perm(c3, K, 0x4342), zz, ss));
+    }
+  }
+}
+
+// Rows of the paper's page. store_row_c4r4 writes one row (64 INT4 codes) of
+// chunk k as RN_f16(s (q - z)) with the stored bf16 (content) or fp32 (RoPE)
+// scale. q - z is exact in fp16 (as in store_row); a bf16 scale in [2^-14,
+// 65504] is an fp16 value, so the fp16 product is the single rounding of the
+// exact product. Any other scale (the fp32 RoPE scale, a tiny or huge content
+// scale) multiplies in fp32 and rounds to fp16 after (store_row_c4r4_f32): one
+// rounding for content, whose fp32 product is exact, and
+// RN_f16(RN_f32(s (q - z))) for the RoPE key.
+__device__ __forceinline__ void store_row_c4r4_f32(uint32_t chunk_base, int row, const uint4& a, const uint4& b,
+                                                   float s, uint32_t zz) {
+  constexpr uint32_t K = 0x64646464u;
+  const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+  auto dqf = [&](uint32_t x) {
+    uint32_t t;
+    asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(t) : "r"(x), "r"(zz));
+    const float2 d = __half22float2(*reinterpret_cast<const __half2*>(&t));
+    return pack_h2(d.x * s, d.y * s);
+  };
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const uint32_t lo = w[i] & 0x0F0F0F0Fu;
+    const uint32_t hi = (w[i] >> 4) & 0x0F0F0F0Fu;
+    sts_v4(chunk_base + swz_off(row, i, 128), dqf(__byte_perm(lo, K, 0x4140)), dqf(__byte_perm(hi, K, 0x4140)),
+           dqf(__byte_perm(lo, K, 0x4342)), dqf(__byte_perm(hi, K, 0x4342)));
+  }
+}
+
+template <bool kContent>
+__device__ __forceinline__ void store_row_c4r4(uint32_t chunk_base, int row, const Fetch& f) {
+  if (!f.ok) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) sts_v4(chunk_base + swz_off(row, i, 128), 0, 0, 0, 0);
+    return;
+  }
+  const float s = __uint_as_float(f.sz);
+  const __half2 zz2 = __half2half2(__float2half_rn(1024.0f + static_cast<float>(f.z)));
+  const uint32_t zz = *reinterpret_cast<const uint32_t*>(&zz2);
+  if constexpr (!kContent) {
+    store_row_c4r4_f32(chunk_base, row, f.a, f.b, s, zz);
+  } else {
+    const __half sh = __float2half_rn(s);
+    if (__half2float(sh) != s) {  // only a content scale outside fp16's normal range
+      store_row_c4r4_f32(chunk_base, row, f.a, f.b, s, zz);
+      return;
+    }
+    const __half2 s2 = __half2half2(sh);
+    const uint32_t ss = *reinterpret_cast<const uint32_t*>(&s2);
+    constexpr uint32_t K = 0x64646464u;
+    const uint32_t w[8] = {f.a.x, f.a.y, f.a.z, f.a.w, f.b.x, f.b.y, f.b.z, f.b.w};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t lo = w[i] & 0x0F0F0F0Fu;
+      const uint32_t hi = (w[i] >> 4) & 0x0F0F0F0Fu;
+      sts_v4(chunk_base + swz_off(row, i, 128), dq2(__byte_perm(lo, K, 0x4140), zz, ss),
+             dq2(__byte_perm(hi, K, 0x4140), zz, ss), dq2(__byte_perm(lo, K, 0x4342), zz, ss),
+             dq2(__byte_perm(hi, K, 0x4342), zz, ss));
     }
   }
 }
@@ -687,7 +765,9 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
                             int lane) {
   using C = Cols<HG>;
   const int q4 = warp & 3;
-  const int par = warp >> 2;  // dequantised chunks k = par, par + 2, ...; heads half `par`
+  // dequantised chunks k = par, par + 2, ...; heads half `par` (the mask tells
+  // the compiler par <= 1, so each unrolled chunk step knows whether k < 8)
+  const int par = (warp >> 2) & 1;
   const int row = q4 * 32 + lane;
   const int slot = row & 63;
   const int cb0 = par * C::kPerWarp;
@@ -796,7 +876,15 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
           for (int i = 0; i < 8; ++i) pv[i] = __ldg(reinterpret_cast<const uint4*>(psrc_cur + k * 128) + i);
           store_row_prot<CB>(chunks + k * kChunkBytes, row, pv, k);
         } else {
-          store_row<CB>(chunks + k * kChunkBytes, row, f[kc], CB == 4 || k == 8);
+          if constexpr (CB == kC4R4) {
+            if (k < 8) {
+              store_row_c4r4<true>(chunks + k * kChunkBytes, row, f[kc]);
+            } else {
+              store_row_c4r4<false>(chunks + k * kChunkBytes, row, f[kc]);
+            }
+          } else {
+            store_row<CB>(chunks + k * kChunkBytes, row, f[kc], CB == 4 || k == 8);
+          }
         }
         f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);  // the next tile's rows of this chunk
       }
@@ -1331,6 +1419,9 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
   prm.trace = nullptr;
 #endif
   const bool prot = prm.prot != nullptr;
+  if (a.cache_kind == kC4R4)
+    return prot ? launch_hg<kC4R4, true>(hg, prm, stream, a.ev_before_main, a.ev_after_main)
+                : launch_hg<kC4R4, false>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
   if (a.cache_kind == 4)
     return prot ? launch_hg<4, true>(hg, prm, stream, a.ev_before_main, a.ev_after_main)
                 : launch_hg<4, false>(hg, prm, stream, a.ev_before_main, a.ev_after_main);

@@ -6,6 +6,7 @@
 
 namespace qmla {
 
+// c_bits: 4 or 2 (this library's block) or kC4R4 (the paper's page).
 cudaError_t launch_quant_append(void* pool, int c_bits, int num_blocks, const uint16_t* latent,
                                 const uint16_t* k_pe, const int32_t* seq_ids,
                                 const int32_t* positions, int n, const int32_t* table, int num_seqs,
@@ -28,7 +29,7 @@ DecodeWorkspace decode_workspace_layout(int batch, int heads, int grid);
 
 struct DecodeArgs {
   const void* pool;
-  int cache_kind;  // 4 or 2: packed content bits; 16: BF16 cache
+  int cache_kind;  // 4 or 2: packed content bits; kC4R4: the paper's page; 16: BF16 cache
   int num_blocks;
   const uint16_t* q_latent;
   const uint16_t* q_pe;

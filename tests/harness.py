@@ -13,6 +13,7 @@ import torch
 import paper_2609_36760_gb300 as Q
 from oracle import attention as OA
 from oracle import layout as OL
+from oracle import paper_format as OF
 from oracle import protection as OP
 from oracle import quantizer as OQ
 from workloads import synthetic as W
@@ -28,11 +29,15 @@ def rel_l2(a, b) -> float:
 
 
 class Case:
-    """A workload materialised on the GPU (packed or BF16 cache) plus its inputs on the host."""
+    """A workload materialised on the GPU (packed or BF16 cache) plus its inputs on the host.
+    c4r4=True stores the packed cache in the paper's page format (INT4 only)."""
 
-    def __init__(self, w: W.Workload, bf16_cache: bool = False, device: str = "cuda", protect: bool = False):
+    def __init__(self, w: W.Workload, bf16_cache: bool = False, device: str = "cuda", protect: bool = False,
+                 c4r4: bool = False):
+        assert not c4r4 or (w.c_bits == 4 and not bf16_cache)
         self.w = w
         self.bf16 = bf16_cache
+        self.c4r4 = c4r4
         self.protect = protect
         self.dev = device
         self.prefill = W.seq_lengths(w)
@@ -41,7 +46,7 @@ class Case:
         self.table = table
         self.nblocks = nblocks
         self.gains = W.channel_gains(w)
-        bb = Q.bf16_block_bytes() if bf16_cache else Q.block_bytes(w.c_bits)
+        bb = Q.bf16_block_bytes() if bf16_cache else (Q.c4r4_page_bytes() if c4r4 else Q.block_bytes(w.c_bits))
         self.pool = torch.full((nblocks, bb), POISON, dtype=torch.uint8, device=device)
         self.table_d = table.to(device)
         self.dev_err = torch.zeros(1, dtype=torch.int32, device=device)
@@ -63,7 +68,11 @@ class Case:
         kpe_d = kpe.contiguous().to(self.dev)
         sid = None if seq_ids is None else torch.as_tensor(seq_ids, dtype=torch.int32).to(self.dev)
         pos = torch.as_tensor(positions, dtype=torch.int32).to(self.dev)
-        if self.protect:
+        if self.c4r4:
+            la = torch.as_tensor(lens_after, dtype=torch.int32).to(self.dev) if self.protect else None
+            Q.quant_append_c4r4(self.pool, lat_d, kpe_d, sid, pos, self.table_d, self.dev_err, seq_lens=la,
+                                prot=self.prot)
+        elif self.protect:
             la = torch.as_tensor(lens_after, dtype=torch.int32).to(self.dev)
             Q.quant_append_protected(self.pool, self.w.c_bits, lat_d, kpe_d, sid, pos, self.table_d, la, self.prot,
                                      self.dev_err)
@@ -116,7 +125,10 @@ class Case:
         ws.fill_(0x7F)
         sl = torch.tensor(lens, dtype=torch.int32, device=self.dev)
         ql_d, qp_d = ql.contiguous().to(self.dev), qp.contiguous().to(self.dev)
-        if self.protect:
+        if self.c4r4:
+            Q.mla_decode_c4r4(self.pool, ql_d, qp_d, self.table_d, sl, TAU, out, lse, ws, self.dev_err,
+                              prot=self.prot if self.protect else None)
+        elif self.protect:
             Q.mla_decode_protected(self.pool, self.w.c_bits, ql_d, qp_d, self.table_d, sl, self.prot, TAU, out, lse,
                                    ws, self.dev_err)
         elif self.bf16:
@@ -136,11 +148,15 @@ class Case:
         kpf = kp[:L].double().numpy()
         if self.bf16:
             return latf, kpf
-        q, s, z = OL.quantize_tokens(latf, kpf, self.w.c_bits)
-        if fp16_tiles:
+        if self.c4r4:
+            q, s, z = OF.quantize_tokens(latf, kpf)
+            C, K = OF.tile_values(q, s, z) if fp16_tiles else OF.dequantize_tokens(q, s, z)
+        elif fp16_tiles:
+            q, s, z = OL.quantize_tokens(latf, kpf, self.w.c_bits)
             x = OQ.dequantize_fp16(q.reshape(L, 9, 64), s, z).astype(np.float64).reshape(L, 576)
             C, K = x[:, :512], x[:, 512:]
         else:
+            q, s, z = OL.quantize_tokens(latf, kpf, self.w.c_bits)
             C, K = OA.dequantize_tokens(q, s, z)
         if self.protect:
             # protected positions attend with the original values (rounded to fp16
@@ -160,13 +176,17 @@ class Case:
 
     def oracle_pool_blocks(self, seqs, upto: list[int]):
         """Oracle-written bytes of the blocks owned by ``seqs`` (tokens [0, upto[b]))."""
-        bb = OL.block_bytes(self.w.c_bits)
+        bb = OF.PAGE_BYTES if self.c4r4 else OL.block_bytes(self.w.c_bits)
         pool = np.full((self.nblocks, bb), POISON, np.uint8)
         for b in seqs:
             lat, kp = self.tokens(b)
             n = upto[b]
-            OL.write_tokens(pool, self.w.c_bits, lat[:n].double().numpy(), kp[:n].double().numpy(),
-                            np.full(n, b), np.arange(n), self.table.numpy())
+            if self.c4r4:
+                OF.write_tokens(pool, lat[:n].double().numpy(), kp[:n].double().numpy(), np.full(n, b),
+                                np.arange(n), self.table.numpy())
+            else:
+                OL.write_tokens(pool, self.w.c_bits, lat[:n].double().numpy(), kp[:n].double().numpy(),
+                                np.full(n, b), np.arange(n), self.table.numpy())
         blocks = sorted({int(x) for b in seqs for x in self.table[b].tolist() if x >= 0})
         return blocks, pool[blocks]
 

@@ -71,3 +71,23 @@ def test_invalid_arguments_are_rejected_before_any_launch(libqmla):
     assert L.qmla_mla_decode(*args) == 1
     assert L.qmla_decode_workspace_bytes(0, 16) == 0
     assert L.qmla_decode_workspace_bytes(1, 0) == 0
+
+
+def test_c4r4_host_checks(libqmla):
+    L = libqmla
+    assert L.qmla_c4r4_page_bytes() == 20480
+    fake = ctypes.c_void_p(0x10000)
+    # protection rows asked for without the lengths after the call
+    assert L.qmla_quant_append_c4r4(fake, 4, fake, fake, None, fake, 1, fake, 1, 1, None, fake, None, None) == 1
+    # misaligned protection buffer
+    assert L.qmla_quant_append_c4r4(fake, 4, fake, fake, None, fake, 1, fake, 1, 1, fake, ctypes.c_void_p(0x10008),
+                                    None, None) == 1
+    # n == 0: nothing to do, nothing touched
+    assert L.qmla_quant_append_c4r4(None, 4, None, None, None, None, 0, None, 1, 1, None, None, None, None) == 0
+    # decode: misaligned protection buffer, null output
+    args = [fake, 4, fake, fake, 1, 16, fake, 1, fake, ctypes.c_void_p(0x10008), 0.1, fake, None, fake, 1 << 30,
+            None, None]
+    assert L.qmla_mla_decode_c4r4(*args) == 1
+    args[9] = None
+    args[11] = None
+    assert L.qmla_mla_decode_c4r4(*args) == 1
