@@ -19,8 +19,10 @@ protection sink4/local128 BF16 protection: the protected set, this library's
 paper_format the paper's own 20,480-byte page: bf16 content scales, fp32 RoPE
            scale, uint8 zero points, its quantiser staging, writer and reader
            (App. C.4, App. C.5 storage layout)
+multi_query decode with T query tokens per sequence: Eq. mla_compact with its
+           additive causal mask, masked partials and their merge (App. C.5)
 
 Every function is pinned by tests under ``tests/test_oracle_*.py``; nothing in
 this package is marked "parity unpinned".
 """
-from . import attention, layout, paper_format, protection, quantizer, storage  # noqa: F401
+from . import attention, layout, multi_query, paper_format, protection, quantizer, storage  # noqa: F401
