@@ -15,6 +15,7 @@ scaling, max time over ranks. `--impl reference` times the CPU oracle instead.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import math
@@ -51,6 +52,9 @@ def parse():
                     help="sink4/local128 BF16 protection (the paper's C4R4 serving configuration)")
     ap.add_argument("--c4r4", action="store_true",
                     help="store the INT4 cache in the paper's own 20,480-byte page (bf16/fp32 scales, uint8 zeros)")
+    ap.add_argument("--q-tokens", type=int, default=1,
+                    help="query tokens per sequence (multi-token prediction / speculative verification); each step "
+                         "appends that many tokens and scores them under the causal mask")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
@@ -72,12 +76,15 @@ def load_peaks():
     return dict(FALLBACK_PEAKS), "fallback"
 
 
-def workload_cost(w: W.Workload, lens: list[int], bf16: bool, c4r4: bool = False):
-    """Algorithmic FLOPs and HBM bytes of one decode launch (see the design notes)."""
+def workload_cost(w: W.Workload, lens: list[int], bf16: bool, c4r4: bool = False, q_tokens: int = 1):
+    """Algorithmic FLOPs and HBM bytes of one decode launch (see the design notes).
+    With T query tokens per sequence every cached token is scored by T x H query
+    rows (the causal mask hides T(T-1)/2 of a sequence's pairs; not subtracted)."""
     tokens = sum(lens)
-    flops = 2.0 * w.heads * (576 + 512) * tokens
+    rows = q_tokens * w.heads
+    flops = 2.0 * rows * (576 + 512) * tokens
     per_tok = 1152 if bf16 else (320 if c4r4 else (324 if w.c_bits == 4 else 196))
-    nbytes = tokens * per_tok + w.batch * w.heads * (576 * 2 + 512 * 4 + 4)
+    nbytes = tokens * per_tok + w.batch * rows * (576 * 2 + 512 * 4 + 4)
     return flops, nbytes
 
 
@@ -159,9 +166,14 @@ class Workspace:
     """GPU state of one workload: pool, block table, per-step inputs."""
 
     def __init__(self, w: W.Workload, bf16: bool, dev: torch.device, nsteps: int, protect: bool = False,
-                 c4r4: bool = False):
+                 c4r4: bool = False, q_tokens: int = 1):
         import paper_2609_36760_gb300 as Q
         self.Q = Q
+        self.q_tokens = q_tokens
+        if q_tokens > 1:
+            if bf16 or c4r4:
+                raise SystemExit("--q-tokens > 1 runs on the INT4/INT2 block (protection optional)")
+            w = dataclasses.replace(w, append=max(w.append, q_tokens))  # the scored tokens are the appended ones
         self.w, self.bf16, self.dev = w, bf16, dev
         self.protect = protect and not bf16
         self.c4r4 = c4r4 and not bf16
@@ -197,7 +209,7 @@ class Workspace:
         self.steps = []
         for s in range(self.nsteps):
             si = self.step_in[s]
-            ql, qp = W.queries(w, s)
+            ql, qp = W.queries(w, s) if q_tokens == 1 else W.queries_multi(w, s, q_tokens)
             lens = [n + w.append * (s + 1) for n in self.prefill]
             host = {
                 "lat": torch.cat(si["lat"]) if si["lat"] else torch.zeros(0, 512, dtype=torch.bfloat16),
@@ -208,9 +220,10 @@ class Workspace:
                 "lens": torch.tensor(lens, dtype=torch.int32),
             }
             self.steps.append({"host": host, "dev": {k: v.to(dev) for k, v in host.items()}, "lens": lens})
-        self.out = torch.empty((w.batch, w.heads, 512), dtype=torch.float32, device=dev)
-        self.lse = torch.empty((w.batch, w.heads), dtype=torch.float32, device=dev)
-        self.ws = Q.workspace_for(w.batch, w.heads, dev)
+        qshape = (w.batch, w.heads) if q_tokens == 1 else (w.batch, q_tokens, w.heads)
+        self.out = torch.empty(qshape + (512,), dtype=torch.float32, device=dev)
+        self.lse = torch.empty(qshape, dtype=torch.float32, device=dev)
+        self.ws = Q.workspace_for(w.batch, q_tokens * w.heads, dev)
 
     def _append(self, lat, kp, sid, pos, lens_after=None):
         if lat.shape[0] == 0:
@@ -231,7 +244,10 @@ class Workspace:
         out = self.out if out is None else out
         lse = self.lse if lse is None else lse
         self._append(d["lat"], d["kp"], d["sid"], d["pos"], d["lens"])
-        if self.c4r4:
+        if self.q_tokens > 1:
+            self.Q.mla_decode_multi(self.pool, self.w.c_bits, d["ql"], d["qp"], self.table, d["lens"], TAU, out,
+                                    lse, self.ws, self.err, prot=self.prot)
+        elif self.c4r4:
             self.Q.mla_decode_c4r4(self.pool, d["ql"], d["qp"], self.table, d["lens"], TAU, out, lse, self.ws,
                                    self.err, prot=self.prot)
         elif self.protect:
@@ -259,7 +275,8 @@ def run_native(args, ws_world: int, rank: int, local: int):
         dist.init_process_group("nccl", device_id=dev)
     w = W.WORKLOADS[args.workload]
     K, Wm = args.steps, args.warmup
-    state = Workspace(w, args.bf16_cache, dev, K + Wm, protect=args.protect, c4r4=args.c4r4)
+    state = Workspace(w, args.bf16_cache, dev, K + Wm, protect=args.protect, c4r4=args.c4r4, q_tokens=args.q_tokens)
+    w = state.w
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # larger than the 126 MB L2
     stream = torch.cuda.current_stream(dev)
 
@@ -318,7 +335,7 @@ def run_native(args, ws_world: int, rank: int, local: int):
 
     # roofline of the main decode kernel
     peaks, peak_src = load_peaks()
-    flops, nbytes = workload_cost(w, lens_all[0], args.bf16_cache, state.c4r4)
+    flops, nbytes = workload_cost(w, lens_all[0], args.bf16_cache, state.c4r4, args.q_tokens)
     t_tc = flops / (peaks["bf16_tflops"] * 1e12)
     t_hbm = nbytes / (peaks["hbm_gbs"] * 1e9)
     tensor_bound = t_tc >= t_hbm
@@ -334,7 +351,8 @@ def run_native(args, ws_world: int, rank: int, local: int):
     roof["traffic"] = (prof["dram_bytes_per_launch"] if prof and prof.get("workload") == args.workload
                        and bool(prof.get("bf16_cache")) == bool(args.bf16_cache)
                        and bool(prof.get("protect")) == bool(args.protect)
-                       and bool(prof.get("c4r4")) == bool(state.c4r4) else None)
+                       and bool(prof.get("c4r4")) == bool(state.c4r4)
+                       and int(prof.get("q_tokens", 1)) == args.q_tokens else None)
     roof["kernel"] = "decode_main"
     roof["kernel_us"] = round(ms_main * 1e3, 2)
     roof["algorithmic_flops"] = flops
@@ -352,6 +370,7 @@ def run_native(args, ws_world: int, rank: int, local: int):
         "dtype": "f16", "data": "synthetic (seeded generators, workloads/synthetic.py)",
         "config": {"workload": w.name, "batch_per_gpu": w.batch, "heads": w.heads, "c_bits": w.c_bits,
                    "pe_bits": 4, "cache": cache_name(w, args.bf16_cache, args.protect, state.c4r4),
+                   "q_tokens_per_seq": args.q_tokens,
                    "kv_tokens_per_step_per_gpu": tok_per_step, "l2": "flushed (256 MB write) before every timed step",
                    "parallelism": f"replicas x{ws_world} (independent sequences)"},
         "us_per_step": round(ms_step_max * 1e3, 2),
@@ -363,7 +382,7 @@ def run_native(args, ws_world: int, rank: int, local: int):
     }
     if rank == 0 and ws_world == 1 and not args.no_cpu_baseline:
         res["cpu_baseline"] = cpu_baseline(w, args.bf16_cache, budget_s=15.0, protect=args.protect,
-                                           c4r4=state.c4r4)
+                                           c4r4=state.c4r4, q_tokens=args.q_tokens)
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
@@ -417,18 +436,21 @@ def run_e2e(state: Workspace, K: int, flush, dev, tokens: float, n_world: int, d
 
 # ------------------------------------------------------------------ oracle
 def oracle_step_sample(w: W.Workload, bf16: bool, budget_s: float, max_seqs: int | None = None,
-                       protect: bool = False, c4r4: bool = False):
+                       protect: bool = False, c4r4: bool = False, q_tokens: int = 1):
     """Times the CPU oracle on one decode step (append of the step's tokens,
     read-back and dequantisation of each sequence's cache, fp64 attention) for
     as many sequences as fit in `budget_s`. Returns (tokens, seconds, nseq)."""
     import numpy as np
     from oracle import attention as OA
     from oracle import layout as OL
+    from oracle import multi_query as OM
     from oracle import paper_format as OF
 
+    if q_tokens > 1:
+        w = dataclasses.replace(w, append=max(w.append, q_tokens))
     prefill = W.seq_lengths(w)
     gains = W.channel_gains(w)
-    ql, qp = W.queries(w, 0)
+    ql, qp = W.queries(w, 0) if q_tokens == 1 else W.queries_multi(w, 0, q_tokens)
     tot_tok, tot_s, nseq = 0, 0.0, 0
     limit = w.batch if max_seqs is None else min(max_seqs, w.batch)
     for b in range(limit):
@@ -462,7 +484,10 @@ def oracle_step_sample(w: W.Workload, bf16: bool, budget_s: float, max_seqs: int
             P = OP.protected_positions(L)
             C, K = np.array(C), np.array(K)
             C[P], K[P] = lat[P], kp[P]
-        OA.attend(ql[b].double().numpy(), qp[b].double().numpy(), C, K, TAU)
+        if q_tokens == 1:
+            OA.attend(ql[b].double().numpy(), qp[b].double().numpy(), C, K, TAU)
+        else:
+            OM.attend_multi(ql[b].double().numpy(), qp[b].double().numpy(), C, K, TAU)
         tot_s += time.perf_counter() - t0
         tot_tok += L
         nseq += 1
@@ -478,8 +503,9 @@ def cpu_cores() -> int:
         return os.cpu_count() or 1
 
 
-def cpu_baseline(w: W.Workload, bf16: bool, budget_s: float, protect: bool = False, c4r4: bool = False):
-    tok, sec, nseq = oracle_step_sample(w, bf16, budget_s, protect=protect, c4r4=c4r4)
+def cpu_baseline(w: W.Workload, bf16: bool, budget_s: float, protect: bool = False, c4r4: bool = False,
+                 q_tokens: int = 1):
+    tok, sec, nseq = oracle_step_sample(w, bf16, budget_s, protect=protect, c4r4=c4r4, q_tokens=q_tokens)
     return {"value": round(tok / sec, 1), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
             "sample": f"{nseq} of {w.batch} sequences of one decode step ({tok} KV tokens, "
                       f"{w.heads} heads): append + cache read-back + dequantisation + fp64 attention, "
@@ -494,7 +520,8 @@ def run_reference(args, ws_world: int, rank: int):
     steps = []
     for i in range(args.warmup + args.steps):
         tok, sec, nseq = oracle_step_sample(w, args.bf16_cache, budget_s=1e9, max_seqs=min(4, w.batch),
-                                            protect=args.protect, c4r4=args.c4r4 and not args.bf16_cache)
+                                            protect=args.protect, c4r4=args.c4r4 and not args.bf16_cache,
+                                            q_tokens=args.q_tokens)
         if i >= args.warmup:
             steps.append((tok, sec))
     tok = sum(t for t, _ in steps)
@@ -506,6 +533,7 @@ def run_reference(args, ws_world: int, rank: int):
            "data": "synthetic (seeded generators, workloads/synthetic.py)",
            "config": {"workload": w.name, "batch_per_gpu": w.batch, "heads": w.heads, "c_bits": w.c_bits,
                       "pe_bits": 4, "cache": cache_name(w, args.bf16_cache, args.protect, args.c4r4),
+                      "q_tokens_per_seq": args.q_tokens,
                       "sample_per_step": f"{min(4, w.batch)} sequences"},
            "cpu_baseline": {"value": round(value, 1), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                             "sample": f"{min(4, w.batch)} of {w.batch} sequences per step, {len(steps)} steps"},

@@ -15,6 +15,7 @@
  *                       "global attention normalization")
  *   *_protected         the same with sink4/local128 BF16 protection (App. C.5)
  *   *_c4r4              the same over the paper's own 20,480-byte INT4 page
+ *   qmla_mla_decode_multi  several query tokens per sequence under the causal mask
  *
  * Conventions for every call
  * --------------------------
@@ -81,6 +82,9 @@ enum qmla_device_error {
   QMLA_DEVERR_BAD_SEQ = 4u,       /* an append sequence id outside [0, num_seqs) */
   QMLA_DEVERR_TIMEOUT = 8u        /* an on-chip pipeline wait ran out; that kernel left early */
 };
+
+/* Most query tokens per sequence qmla_mla_decode_multi accepts. */
+#define QMLA_MAX_Q_TOKENS 8
 
 /* Bytes of one 64-token block for content bit width c_bits (4 -> 20736,
  * 2 -> 12544); 0 if c_bits is not supported. */
@@ -151,7 +155,8 @@ int qmla_quant_append_protected(void* pool_dev, int c_bits, int num_blocks, cons
                                 uint32_t* dev_err_dev, qmla_stream_t stream);
 
 /* Workspace bytes qmla_mla_decode needs for this batch and head count on the
- * current device (split plan + split partials). */
+ * current device (split plan + split partials). For qmla_mla_decode_multi pass
+ * heads = q_tokens x heads (up to 128 x QMLA_MAX_Q_TOKENS); 0 for bad arguments. */
 size_t qmla_decode_workspace_bytes(int batch, int heads);
 
 /*
@@ -194,6 +199,35 @@ int qmla_mla_decode_protected(const void* pool_dev, int c_bits, int num_blocks, 
                               int max_blocks, const int32_t* seq_lens_dev, const void* prot_dev,
                               float softmax_scale, float* out_dev, float* lse_dev, void* workspace_dev,
                               size_t workspace_bytes, uint32_t* dev_err_dev, qmla_stream_t stream);
+
+/* Decode with q_tokens query tokens per sequence (multi-token prediction,
+ * speculative verification): Eq. mla_compact with its additive causal mask.
+ * For sequence b with L = seq_lens_dev[b] cached tokens (the q_tokens new ones
+ * included, written by the append beforehand), query token t sits at position
+ * L - q_tokens + t and attends to positions [0, L - q_tokens + t]:
+ *     S[b,t,h,p] = softmax_scale * (q_latent[b,t,h,:] . C_hat[b,p,:] + q_pe[b,t,h,:] . K_hat[b,p,:]),
+ *                  p <= L - q_tokens + t
+ *     out[b,t,h,:] = sum_p softmax_p(S[b,t,h,:]) C_hat[b,p,:];  lse[b,t,h] = log sum_p exp(S[b,t,h,p])
+ * A query token with no admissible position (L - q_tokens + t < 0) gets out = 0,
+ * lse = -inf. One pass over each sequence's cache serves all its query tokens:
+ * the kernel treats the q_tokens x heads (token, head) pairs as heads.
+ *
+ *   q_latent_dev    [batch, q_tokens, heads, 512] bf16, 16-byte aligned
+ *   q_pe_dev        [batch, q_tokens, heads, 64]  bf16, 16-byte aligned
+ *   q_tokens        1 .. QMLA_MAX_Q_TOKENS; heads 1..128 per token
+ *   prot_dev        NULL, or the sink4/local128 protection buffer (as
+ *                   qmla_mla_decode_protected; P_L from the full length L)
+ *   out_dev         [batch, q_tokens, heads, 512] float32
+ *   lse_dev         [batch, q_tokens, heads] float32, or NULL
+ *   workspace_dev   >= qmla_decode_workspace_bytes(batch, q_tokens * heads)
+ * Other arguments, ownership and errors as qmla_mla_decode; q_tokens = 1 is
+ * qmla_mla_decode. */
+int qmla_mla_decode_multi(const void* pool_dev, int c_bits, int num_blocks, const uint16_t* q_latent_dev,
+                          const uint16_t* q_pe_dev, int batch, int q_tokens, int heads,
+                          const int32_t* block_table_dev, int max_blocks, const int32_t* seq_lens_dev,
+                          const void* prot_dev, float softmax_scale, float* out_dev, float* lse_dev,
+                          void* workspace_dev, size_t workspace_bytes, uint32_t* dev_err_dev,
+                          qmla_stream_t stream);
 
 /* The same decode over the BF16 comparison cache (same kernel, no dequantisation;
  * the paper's BF16 baseline, App. F.1). */

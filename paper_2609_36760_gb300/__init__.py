@@ -73,6 +73,9 @@ def lib():
     L.qmla_mla_decode_protected.argtypes = [vp, i32, i32, vp, vp, i32, i32, vp, i32, vp, vp, f32, vp, vp, vp, sz,
                                             vp, vp]
     L.qmla_mla_decode_protected.restype = i32
+    L.qmla_mla_decode_multi.argtypes = [vp, i32, i32, vp, vp, i32, i32, i32, vp, i32, vp, vp, f32, vp, vp, vp, sz,
+                                        vp, vp]
+    L.qmla_mla_decode_multi.restype = i32
     L.qmla_c4r4_page_bytes.argtypes, L.qmla_c4r4_page_bytes.restype = [], sz
     L.qmla_quant_append_c4r4.argtypes = [vp, i32, vp, vp, vp, vp, i32, vp, i32, i32, vp, vp, vp, vp]
     L.qmla_quant_append_c4r4.restype = i32
@@ -179,6 +182,20 @@ def mla_decode_protected(pool: torch.Tensor, c_bits: int, q_latent: torch.Tensor
                                          workspace.numel() * workspace.element_size(), _ptr(dev_err),
                                          _stream(stream))
     _check("qmla_mla_decode_protected", st)
+
+
+def mla_decode_multi(pool: torch.Tensor, c_bits: int, q_latent: torch.Tensor, q_pe: torch.Tensor,
+                     block_table: torch.Tensor, seq_lens: torch.Tensor, softmax_scale: float, out: torch.Tensor,
+                     lse: torch.Tensor | None, workspace: torch.Tensor, dev_err: torch.Tensor,
+                     prot: torch.Tensor | None = None, stream=None) -> None:
+    """qmla_mla_decode_multi: q_latent bf16 [B,T,H,512], q_pe bf16 [B,T,H,64],
+    out f32 [B,T,H,512], lse f32 [B,T,H]; workspace for B x (T*H) heads."""
+    B, T, H = q_latent.shape[0], q_latent.shape[1], q_latent.shape[2]
+    st = lib().qmla_mla_decode_multi(_ptr(pool), c_bits, pool.shape[0], _ptr(q_latent), _ptr(q_pe), B, T, H,
+                                     _ptr(block_table), block_table.shape[1], _ptr(seq_lens), _ptr(prot),
+                                     float(softmax_scale), _ptr(out), _ptr(lse), _ptr(workspace),
+                                     workspace.numel() * workspace.element_size(), _ptr(dev_err), _stream(stream))
+    _check("qmla_mla_decode_multi", st)
 
 
 def c4r4_page_bytes() -> int:

@@ -59,15 +59,18 @@ int append_common_checks(const void* pool, int num_blocks, const uint16_t* laten
   return QMLA_OK;
 }
 
+// heads counts every query row of a sequence (q_tokens x heads per token).
 int decode_common(const void* pool, int kind, int num_blocks, const uint16_t* q_latent, const uint16_t* q_pe,
                   int batch, int heads, const int32_t* table, int max_blocks, const int32_t* seq_lens,
                   float softmax_scale, float* out, float* lse, void* workspace, size_t workspace_bytes,
-                  uint32_t* dev_err, qmla_stream_t stream, const void* prot = nullptr) {
+                  uint32_t* dev_err, qmla_stream_t stream, const void* prot = nullptr, int q_tokens = 1) {
   if (pool == nullptr || q_latent == nullptr || q_pe == nullptr || table == nullptr || seq_lens == nullptr ||
       out == nullptr || workspace == nullptr)
     return QMLA_ERR_INVALID_ARG;
   if (prot != nullptr && !aligned(prot, 16)) return QMLA_ERR_INVALID_ARG;
-  if (batch <= 0 || heads < 1 || heads > 128 || num_blocks <= 0 || max_blocks <= 0) return QMLA_ERR_INVALID_ARG;
+  if (q_tokens < 1 || q_tokens > QMLA_MAX_Q_TOKENS || heads % q_tokens != 0) return QMLA_ERR_INVALID_ARG;
+  if (batch <= 0 || heads < 1 || heads / q_tokens > 128 || num_blocks <= 0 || max_blocks <= 0)
+    return QMLA_ERR_INVALID_ARG;
   if (!(softmax_scale > 0.0f) || softmax_scale > 1e30f) return QMLA_ERR_INVALID_ARG;
   if (!aligned(pool, 16) || !aligned(q_latent, 16) || !aligned(q_pe, 16) || !aligned(table, 4) ||
       !aligned(seq_lens, 4) || !aligned(out, 16) || (lse != nullptr && !aligned(lse, 4)) ||
@@ -97,6 +100,7 @@ int decode_common(const void* pool, int kind, int num_blocks, const uint16_t* q_
   a.dev_err = dev_err;
   a.grid = di.sms;
   a.prot = prot;
+  a.q_tokens = q_tokens;
   a.ev_before_main = g_ev_before_main;
   a.ev_after_main = g_ev_after_main;
   cudaError_t e = qmla::launch_decode(a, reinterpret_cast<cudaStream_t>(stream));
@@ -175,7 +179,7 @@ int qmla_bf16_append(void* pool_dev, int num_blocks, const uint16_t* latent_dev,
 }
 
 size_t qmla_decode_workspace_bytes(int batch, int heads) {
-  if (batch <= 0 || heads < 1 || heads > 128) return 0;
+  if (batch <= 0 || heads < 1 || heads > 128 * QMLA_MAX_Q_TOKENS) return 0;
   DevInfo di;
   if (current_device_info(di) != QMLA_OK) return 0;
   return qmla::decode_workspace_layout(batch, heads, di.sms).total;
@@ -235,6 +239,18 @@ int qmla_mla_decode_c4r4(const void* pool_dev, int num_blocks, const uint16_t* q
   return decode_common(pool_dev, qmla::kC4R4, num_blocks, q_latent_dev, q_pe_dev, batch, heads, block_table_dev,
                        max_blocks, seq_lens_dev, softmax_scale, out_dev, lse_dev, workspace_dev, workspace_bytes,
                        dev_err_dev, stream, prot_dev);
+}
+
+int qmla_mla_decode_multi(const void* pool_dev, int c_bits, int num_blocks, const uint16_t* q_latent_dev,
+                          const uint16_t* q_pe_dev, int batch, int q_tokens, int heads,
+                          const int32_t* block_table_dev, int max_blocks, const int32_t* seq_lens_dev,
+                          const void* prot_dev, float softmax_scale, float* out_dev, float* lse_dev,
+                          void* workspace_dev, size_t workspace_bytes, uint32_t* dev_err_dev, qmla_stream_t stream) {
+  if (c_bits != 4 && c_bits != 2) return QMLA_ERR_INVALID_ARG;
+  if (q_tokens < 1 || q_tokens > QMLA_MAX_Q_TOKENS || heads < 1 || heads > 128) return QMLA_ERR_INVALID_ARG;
+  return decode_common(pool_dev, c_bits, num_blocks, q_latent_dev, q_pe_dev, batch, q_tokens * heads,
+                       block_table_dev, max_blocks, seq_lens_dev, softmax_scale, out_dev, lse_dev, workspace_dev,
+                       workspace_bytes, dev_err_dev, stream, prot_dev, q_tokens);
 }
 
 int qmla_mla_decode_bf16cache(const void* pool_dev, int num_blocks, const uint16_t* q_latent_dev,

@@ -88,7 +88,10 @@ struct Params {
   int num_blocks;
   const __nv_bfloat16* q_lat;
   const __nv_bfloat16* q_pe;
+  // heads = q_tokens * hpt "virtual heads" (query token t, head h) -> t * hpt + h;
+  // one query token per sequence: q_tokens = 1, hpt = heads.
   int batch, heads, n_hg;
+  int q_tokens, hpt;
   const int32_t* table;
   int max_blocks;
   const int32_t* seq_lens;
@@ -283,7 +286,7 @@ struct Sched {
 };
 
 struct TileInfo {
-  int b, hg, j, ntok;
+  int b, hg, j, ntok, len;
   bool first, last;
 };
 // Segment position of the current tile, from the schedule alone (no loads).
@@ -301,7 +304,8 @@ __device__ __forceinline__ TileInfo tile_info(const Sched& s, const Params& p) {
   ti.b = s.u / p.n_hg;
   ti.hg = s.u - ti.b * p.n_hg;
   ti.j = s.t - s.pu0;
-  ti.ntok = min(kTileTokens, p.seq_lens[ti.b] - kTileTokens * ti.j);
+  ti.len = p.seq_lens[ti.b];
+  ti.ntok = min(kTileTokens, ti.len - kTileTokens * ti.j);
   ti.first = (s.t == s.t0) || (ti.j == 0);
   ti.last = (s.t + 1 == s.t1) || (s.t + 1 == s.pu1);
   return ti;
@@ -620,9 +624,14 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
+// A thread's row admits the warp's head columns i >= lim (lim = kPerWarp for a
+// row past the sequence end; with several query tokens per sequence, the
+// heads of earlier query tokens do not see the last positions: Eq. mla_compact's
+// causal mask, see row_limit).
+
 // Tile max of the scaled scores of this warp's heads over its 32 rows into red_q[h].
 template <int HG>
-__device__ __forceinline__ void warp_tile_max(uint32_t t_s, float sl2, bool valid, float* red_q, int lane) {
+__device__ __forceinline__ void warp_tile_max(uint32_t t_s, float sl2, int lim, float* red_q, int lane) {
   using C = Cols<HG>;
 #pragma unroll
   for (int c = 0; c < C::kN; ++c) {
@@ -631,7 +640,7 @@ __device__ __forceinline__ void warp_tile_max(uint32_t t_s, float sl2, bool vali
     tmem_ld_wait();
 #pragma unroll
     for (int jj = 0; jj < C::kW; ++jj) {
-      const float x = valid ? __uint_as_float(r[jj]) * sl2 : -INFINITY;
+      const float x = c * C::kW + jj >= lim ? __uint_as_float(r[jj]) * sl2 : -INFINITY;
       const float mx = warp_max_f32(x);
       if (lane == jj) red_q[c * C::kW + jj] = mx;
     }
@@ -641,7 +650,7 @@ __device__ __forceinline__ void warp_tile_max(uint32_t t_s, float sl2, bool vali
 // P^T[t, h] = 2^(S * scale * log2e - m_ref[h]) in fp16 for this warp's heads,
 // into row t of the P tile and into pk; returns whether a weight exceeds 2^8.
 template <int HG>
-__device__ __forceinline__ bool compute_p(uint32_t t_s, const float* mr, float sl2, bool valid, uint32_t ptile,
+__device__ __forceinline__ bool compute_p(uint32_t t_s, const float* mr, float sl2, int lim, uint32_t ptile,
                                           int row, int piece0, uint32_t (&pk)[Cols<HG>::kPerWarp / 2]) {
   using C = Cols<HG>;
   constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
@@ -664,8 +673,9 @@ __device__ __forceinline__ bool compute_p(uint32_t t_s, const float* mr, float s
     for (int jj = 0; jj < C::kW; jj += 2) {
       const float x0 = __uint_as_float(r[jj]) * sl2 - m[jj];
       const float x1 = __uint_as_float(r[jj + 1]) * sl2 - m[jj + 1];
-      over |= valid && (fmaxf(x0, x1) > kRescaleLog2);
-      pk[c * (C::kW / 2) + (jj >> 1)] = valid ? pack_h2(ex2_approx(x0), ex2_approx(x1)) : 0u;
+      const bool ok0 = c * C::kW + jj >= lim, ok1 = c * C::kW + jj + 1 >= lim;
+      over |= (ok0 && x0 > kRescaleLog2) || (ok1 && x1 > kRescaleLog2);
+      pk[c * (C::kW / 2) + (jj >> 1)] = pack_h2(ok0 ? ex2_approx(x0) : 0.0f, ok1 ? ex2_approx(x1) : 0.0f);
     }
 #pragma unroll
     for (int pc = 0; pc < C::kW / 8; ++pc) {
@@ -674,6 +684,21 @@ __device__ __forceinline__ bool compute_p(uint32_t t_s, const float* mr, float s
     }
   }
   return over;
+}
+
+// lim of a tile row: kPerWarp past the sequence end; else the number of this
+// warp's head columns whose query token precedes the row's position. Query
+// token t of a sequence of len tokens sits at position len - q_tokens + t and
+// sees positions <= its own, so row position pos is hidden from tokens
+// t < d = pos - (len - q_tokens), i.e. from virtual heads v < d * hpt: a prefix
+// of the head columns.
+template <int HG>
+__device__ __forceinline__ int row_limit(const Params& p, const TileInfo& ti, int row, int cb0) {
+  constexpr int kPer = Cols<HG>::kPerWarp;
+  if (row >= ti.ntok) return kPer;
+  const int d = kTileTokens * ti.j + row - (ti.len - p.q_tokens);
+  if (d <= 0) return 0;
+  return min(max(d * p.hpt - (ti.hg * HG + cb0), 0), kPer);
 }
 
 // What a segment end needs once its last PV has completed.
@@ -710,7 +735,7 @@ __device__ bool epilogue(const Params& p, const SegEnd& e, Ctrl& ctl, uint32_t t
   if (tid < HG) {
     const float l = (ctl.red[0][tid] + ctl.red[1][tid]) + (ctl.red[2][tid] + ctl.red[3][tid]);
     ctl.alpha[tid] = l;
-    ctl.inv[tid] = 1.0f / l;  // one division per head; the rows below are multiplied
+    ctl.inv[tid] = l > 0.0f ? 1.0f / l : 0.0f;  // one division per head; 0 for a head that saw no key
   }
   if (!group_sync(ctl, gph, p.dev_err)) return false;
   const int h0 = e.hg * HG;
@@ -901,7 +926,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     nx = nn;
     ref_nx = ref_nn;
     const TileInfo ti = tile_info(sc, p);  // ntok of this tile for the softmax (loaded long ago)
-    const bool valid = row < ti.ntok;
+    const int lim = row_limit<HG>(p, ti, row, cb0);
 
     // ---- the previous segment's results (its last PV completed: chunks 6..8 were waited for)
     if (pending) {
@@ -917,7 +942,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     if (lane == 0 && warp == 0) QMLA_TRACE(16, it);
     if (ti.first) {
       // New segment: the reference is this tile's max.
-      warp_tile_max<HG>(t_s, sl2, valid, &ctl.red[q4][cb0], lane);
+      warp_tile_max<HG>(t_s, sl2, lim, &ctl.red[q4][cb0], lane);
       if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
       if (threadIdx.x < HG) {
         const int h = threadIdx.x;
@@ -926,7 +951,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
     }
     uint32_t pk[C::kPerWarp / 2];
-    const bool over = compute_p<HG>(t_s, ctl.m_ref + cb0, sl2, valid, ptile, row, piece0, pk);
+    const bool over = compute_p<HG>(t_s, ctl.m_ref + cb0, sl2, lim, ptile, row, piece0, pk);
     // A weight above 2^8 anywhere in the tile asks for a rescale; the flag is
     // written before p_full, so whoever has seen p_full complete reads it.
     if (__any_sync(0xffffffffu, over) && lane == 0) *reinterpret_cast<volatile uint32_t*>(&ctl.resc_tile) = it + 1;
@@ -944,14 +969,14 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       // The previous PV has completed (its slots were waited for above); the
       // MMA thread waits on p_fixed before this tile's PV.
       tc_fence_after();
-      warp_tile_max<HG>(t_s, sl2, valid, &ctl.red[q4][cb0], lane);
+      warp_tile_max<HG>(t_s, sl2, lim, &ctl.red[q4][cb0], lane);
       if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
       if (threadIdx.x < HG) {
         const int h = threadIdx.x;
         const float mt = fmaxf(fmaxf(ctl.red[0][h], ctl.red[1][h]), fmaxf(ctl.red[2][h], ctl.red[3][h]));
         const float mo = ctl.m_ref[h];
         const float mn = fmaxf(mo, mt);
-        ctl.alpha[h] = exp2f(mo - mn);
+        ctl.alpha[h] = mo == mn ? 1.0f : exp2f(mo - mn);  // also when no key was seen yet (-inf)
         ctl.m_ref[h] = mn;
       }
       if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
@@ -972,7 +997,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
         }
         tmem_st_wait();
       }
-      compute_p<HG>(t_s, ctl.m_ref + cb0, sl2, valid, ptile, row, piece0, pk);
+      compute_p<HG>(t_s, ctl.m_ref + cb0, sl2, lim, ptile, row, piece0, pk);
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
@@ -1313,7 +1338,8 @@ __global__ void __launch_bounds__(128) combine_kernel(const Params p) {
 #pragma unroll
     for (int v = 0; v < 4; ++v) ov[v] = o[v];
     const float Mn = fmaxf(M, ml.x);
-    const float a = exp2f(M - Mn), w = exp2f(ml.x - Mn);
+    // A partial that saw no key for this head has m = -inf and l = o = 0.
+    const float a = M == Mn ? 1.0f : exp2f(M - Mn), w = ml.x == Mn ? 1.0f : exp2f(ml.x - Mn);
     l = l * a + w * ml.y;
 #pragma unroll
     for (int v = 0; v < 4; ++v) {
@@ -1324,7 +1350,7 @@ __global__ void __launch_bounds__(128) combine_kernel(const Params p) {
     }
     M = Mn;
   }
-  const float inv = 1.0f / l;
+  const float inv = l > 0.0f ? 1.0f / l : 0.0f;
 #pragma unroll
   for (int v = 0; v < 4; ++v) out[v] = make_float4(acc[v].x * inv, acc[v].y * inv, acc[v].z * inv, acc[v].w * inv);
   if (lane == 0 && p.lse != nullptr) p.lse[static_cast<size_t>(b) * p.heads + h0 + h] = (M + log2f(l)) * kLn2;
@@ -1397,6 +1423,8 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
   prm.batch = a.batch;
   prm.heads = a.heads;
   prm.n_hg = (a.heads + hg - 1) / hg;
+  prm.q_tokens = a.q_tokens;
+  prm.hpt = a.heads / a.q_tokens;
   prm.table = a.table;
   prm.max_blocks = a.max_blocks;
   prm.seq_lens = a.seq_lens;

@@ -33,7 +33,8 @@ struct DecodeArgs {
   int num_blocks;
   const uint16_t* q_latent;
   const uint16_t* q_pe;
-  int batch, heads;
+  int batch, heads;  // heads: all query rows of a sequence (q_tokens x heads per token)
+  int q_tokens = 1;  // query tokens per sequence (the last q_tokens positions, causal among them)
   const int32_t* table;
   int max_blocks;
   const int32_t* seq_lens;

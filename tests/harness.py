@@ -13,6 +13,7 @@ import torch
 import paper_2609_36760_gb300 as Q
 from oracle import attention as OA
 from oracle import layout as OL
+from oracle import multi_query as OM
 from oracle import paper_format as OF
 from oracle import protection as OP
 from oracle import quantizer as OQ
@@ -137,6 +138,28 @@ class Case:
             Q.mla_decode(self.pool, self.w.c_bits, ql_d, qp_d, self.table_d, sl, TAU, out, lse, ws, self.dev_err)
         torch.cuda.synchronize()
         return out.cpu().numpy(), lse.cpu().numpy()
+
+    def decode_multi(self, step: int, q_tokens: int, lens: list[int] | None = None):
+        """mla_decode_multi with T = q_tokens query tokens per sequence (the last
+        T positions of each sequence): (out [B,T,H,512], lse [B,T,H]) on the host."""
+        ql, qp = W.queries_multi(self.w, step, q_tokens)
+        lens = self.lengths_at(step) if lens is None else lens
+        B, H = self.w.batch, self.w.heads
+        out = torch.full((B, q_tokens, H, 512), float("nan"), dtype=torch.float32, device=self.dev)
+        lse = torch.full((B, q_tokens, H), float("nan"), dtype=torch.float32, device=self.dev)
+        ws = Q.workspace_for(B, q_tokens * H, self.dev)
+        ws.fill_(0x7F)
+        sl = torch.tensor(lens, dtype=torch.int32, device=self.dev)
+        Q.mla_decode_multi(self.pool, self.w.c_bits, ql.contiguous().to(self.dev), qp.contiguous().to(self.dev),
+                           self.table_d, sl, TAU, out, lse, ws, self.dev_err,
+                           prot=self.prot if self.protect else None)
+        torch.cuda.synchronize()
+        return out.cpu().numpy(), lse.cpu().numpy()
+
+    def oracle_decode_multi(self, b: int, L: int, step: int, q_tokens: int, fp16_tiles: bool = False):
+        ql, qp = W.queries_multi(self.w, step, q_tokens)
+        C, K = self.oracle_cache(b, L, fp16_tiles)
+        return OM.attend_multi(ql[b].double().numpy(), qp[b].double().numpy(), C, K, TAU)
 
     def dev_error(self) -> int:
         return Q.read_dev_err(self.dev_err)

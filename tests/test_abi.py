@@ -91,3 +91,17 @@ def test_c4r4_host_checks(libqmla):
     args[9] = None
     args[11] = None
     assert L.qmla_mla_decode_c4r4(*args) == 1
+
+
+def test_multi_query_host_checks(libqmla):
+    L = libqmla
+    assert L.qmla_decode_workspace_bytes(2, 128 * 8 + 1) == 0   # beyond 8 tokens x 128 heads
+    fake = ctypes.c_void_p(0x10000)
+    base = [fake, 4, 4, fake, fake, 1, 2, 16, fake, 1, fake, None, 0.1, fake, None, fake, 1 << 30, None, None]
+    for i, bad in ((6, 0), (6, 9), (7, 0), (7, 129), (1, 3)):   # q_tokens, heads, c_bits
+        args = list(base)
+        args[i] = bad
+        assert L.qmla_mla_decode_multi(*args) == 1, (i, bad)
+    args = list(base)
+    args[11] = ctypes.c_void_p(0x10008)                          # misaligned protection buffer
+    assert L.qmla_mla_decode_multi(*args) == 1

@@ -2,7 +2,7 @@
 
 The paper measures its native backend on synthetic BF16 queries and cache
 values (App. F.1) with d_c = 512, d_r = 64, 64-token pages and one query token
-per sequence. The five workloads below fix batch, heads, context lengths,
+per sequence (``queries_multi`` gives several, for multi-token decoding). The five workloads below fix batch, heads, context lengths,
 bit widths and value distributions; every tensor is drawn from a
 ``torch.Generator`` on the CPU, so a given (workload, sequence) pair always
 yields the same bytes on any machine.
@@ -136,6 +136,14 @@ def queries(w: Workload, step: int = 0) -> tuple[torch.Tensor, torch.Tensor]:
     ql = torch.randn(w.batch, w.heads, D_C, generator=g, dtype=torch.float64) / math.sqrt(D_C)
     qp = torch.randn(w.batch, w.heads, D_R, generator=g, dtype=torch.float64) / math.sqrt(D_R)
     return ql.to(torch.bfloat16), qp.to(torch.bfloat16)
+
+
+def queries_multi(w: Workload, step: int, q_tokens: int) -> tuple[torch.Tensor, torch.Tensor]:
+    """(q_latent [B,T,H,512], q_pe [B,T,H,64]) bf16 for a step that scores T new
+    tokens per sequence: query token t is the single-token query of step
+    step * T + t, so T = 1 gives queries(w, step)."""
+    qs = [queries(w, step * q_tokens + t) for t in range(q_tokens)]
+    return torch.stack([q[0] for q in qs], 1), torch.stack([q[1] for q in qs], 1)
 
 
 def block_table(w: Workload) -> tuple[torch.Tensor, int]:
