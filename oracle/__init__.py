@@ -21,8 +21,11 @@ paper_format the paper's own 20,480-byte page: bf16 content scales, fp32 RoPE
            (App. C.4, App. C.5 storage layout)
 multi_query decode with T query tokens per sequence: Eq. mla_compact with its
            additive causal mask, masked partials and their merge (App. C.5)
+fusion     offline-fusion identities: content rotation/scale with compensated
+           consumers (Eq. content_transform, App. C.1), Prop. 1's reciprocal
+           RoPE-pair transform and its commutation with RoPE (App. C.2)
 
 Every function is pinned by tests under ``tests/test_oracle_*.py``; nothing in
 this package is marked "parity unpinned".
 """
-from . import attention, layout, multi_query, paper_format, protection, quantizer, storage  # noqa: F401
+from . import attention, fusion, layout, multi_query, paper_format, protection, quantizer, storage  # noqa: F401
