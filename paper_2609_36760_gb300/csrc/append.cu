@@ -3,10 +3,12 @@
 // insertion) for this library's block and for the paper's own page, and the
 // plain BF16 writer for the comparison cache.
 //
-// One warp per token. For each of the 9 groups of 64 coordinates, lane l holds
-// coordinates 2l and 2l+1; the group extrema come from warp reductions, every
-// lane quantises its two values, and the packed code words are assembled with
-// shuffles and stored by the lanes that own them.
+// One warp per (token, group): the 9 groups of 64 coordinates of a token are
+// quantised by 9 independent warps, so a decode step's few tokens are not a
+// chain of 9 dependent reductions. Lane l holds coordinates 2l and 2l+1 of its
+// group; the extrema come from warp reductions, every lane quantises its two
+// values, and the packed code words are assembled with shuffles and stored by
+// the lanes that own them.
 #include <cuda_runtime.h>
 
 #include "common.cuh"
@@ -113,55 +115,56 @@ __global__ void __launch_bounds__(256) quant_append_kernel(
     const int32_t* __restrict__ positions, int n, const int32_t* __restrict__ table, int num_seqs,
     int max_blocks, uint32_t* dev_err, uint4* __restrict__ prot, const int32_t* __restrict__ lens) {
   using L = BlockLayout<CB>;
-  const int tok = static_cast<int>((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+  const long long wid = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
-  if (tok >= n) return;
+  if (wid >= static_cast<long long>(n) * kGroups) return;
+  const int tok = static_cast<int>(wid / kGroups);
+  const int g = static_cast<int>(wid - static_cast<long long>(tok) * kGroups);
+  // Quantise first: the group's loads and arithmetic do not wait for the
+  // dependent seq_ids -> block-table lookup, which only the stores need.
+  const int bits = g < 8 ? (CB == kC4R4 ? 4 : CB) : kPeBits;
+  const int m = (1 << bits) - 1;
+  const __nv_bfloat162 v = g < 8 ? latent[static_cast<size_t>(tok) * (kDc / 2) + g * 32 + lane]
+                                 : k_pe[static_cast<size_t>(tok) * (kDr / 2) + lane];
+  const float x0 = __low2float(v), x1 = __high2float(v);
+  const float xmin = warp_min_f32(fminf(x0, x1));
+  const float xmax = warp_max_f32(fmaxf(x0, x1));
+  float s, z;
+  if constexpr (CB == kC4R4) {
+    paper_scale(xmin, xmax, g < 8, s, z);
+  } else {
+    group_scale(xmin, xmax, m, s, z);
+  }
+  const uint32_t code = quant_code(x0, s, z, m) | (quant_code(x1, s, z, m) << bits);
+  // Lane l's 2*bits bits sit at bit offset 2*bits*l of the group's code string.
+  const int lane_bits = 2 * bits;
+  const int lanes_per_word = 32 / lane_bits;
+  uint32_t word = code << ((lane % lanes_per_word) * lane_bits);
+  for (int off = 1; off < lanes_per_word; off <<= 1) word |= __shfl_xor_sync(0xffffffffu, word, off);
+
   int slot = 0;
+  // errors are reported once per token, by its group-0 warp
   uint8_t* blk = token_block(pool, L::kBytes, num_blocks, seq_ids, positions, tok, table, num_seqs,
-                             max_blocks, lane == 0 ? dev_err : nullptr, slot);
+                             max_blocks, lane == 0 && g == 0 ? dev_err : nullptr, slot);
   if (blk == nullptr) return;
-  if (prot != nullptr) {
+  if (prot != nullptr && g == 0) {
     const int seq = seq_ids != nullptr ? seq_ids[tok] : tok;
     protect_row(prot, reinterpret_cast<const uint4*>(latent), reinterpret_cast<const uint4*>(k_pe), tok, seq,
                 positions[tok], lens[seq], lane);
   }
-
-#pragma unroll 1
-  for (int g = 0; g < kGroups; ++g) {
-    const int bits = g < 8 ? (CB == kC4R4 ? 4 : CB) : kPeBits;
-    const int m = (1 << bits) - 1;
-    const __nv_bfloat162 v = g < 8 ? latent[static_cast<size_t>(tok) * (kDc / 2) + g * 32 + lane]
-                                   : k_pe[static_cast<size_t>(tok) * (kDr / 2) + lane];
-    const float x0 = __low2float(v), x1 = __high2float(v);
-    const float xmin = warp_min_f32(fminf(x0, x1));
-    const float xmax = warp_max_f32(fmaxf(x0, x1));
-    float s, z;
+  if (lane % lanes_per_word == 0) {
+    reinterpret_cast<uint32_t*>(blk + L::code_off(g, slot))[lane / lanes_per_word] = word;
+  }
+  if (lane == 0) {
     if constexpr (CB == kC4R4) {
-      paper_scale(xmin, xmax, g < 8, s, z);
-    } else {
-      group_scale(xmin, xmax, m, s, z);
-    }
-    const uint32_t code = quant_code(x0, s, z, m) | (quant_code(x1, s, z, m) << bits);
-    // Lane l's 2*bits bits sit at bit offset 2*bits*l of the group's code string.
-    const int lane_bits = 2 * bits;
-    const int lanes_per_word = 32 / lane_bits;
-    uint32_t word = code << ((lane % lanes_per_word) * lane_bits);
-    for (int off = 1; off < lanes_per_word; off <<= 1) word |= __shfl_xor_sync(0xffffffffu, word, off);
-    if (lane % lanes_per_word == 0) {
-      reinterpret_cast<uint32_t*>(blk + L::code_off(g, slot))[lane / lanes_per_word] = word;
-    }
-    if (lane == 0) {
-      if constexpr (CB == kC4R4) {
-        if (g < 8) {
-          *reinterpret_cast<__nv_bfloat16*>(blk + L::c_scale_off(g, slot)) = __float2bfloat16_rn(s);  // exact
-        } else {
-          *reinterpret_cast<float*>(blk + L::pe_scale_off(slot)) = s;
-        }
-        blk[L::zero_off(g, slot)] = static_cast<uint8_t>(z);
+      if (g < 8) {
+        *reinterpret_cast<__nv_bfloat16*>(blk + L::c_scale_off(g, slot)) = __float2bfloat16_rn(s);  // exact
       } else {
-        *reinterpret_cast<__half2*>(blk + L::sz_off(g, slot)) =
-            __halves2half2(__float2half_rn(s), __float2half_rn(z));
+        *reinterpret_cast<float*>(blk + L::pe_scale_off(slot)) = s;
       }
+      blk[L::zero_off(g, slot)] = static_cast<uint8_t>(z);
+    } else {
+      *reinterpret_cast<__half2*>(blk + L::sz_off(g, slot)) = __halves2half2(__float2half_rn(s), __float2half_rn(z));
     }
   }
 }
@@ -192,7 +195,7 @@ cudaError_t launch_quant_append(void* pool, int c_bits, int num_blocks, const ui
                                 const int32_t* lens) {
   if (n == 0) return cudaSuccess;
   const dim3 block(256);
-  const dim3 grid(static_cast<unsigned>((static_cast<long long>(n) * 32 + 255) / 256));
+  const dim3 grid(static_cast<unsigned>((static_cast<long long>(n) * kGroups * 32 + 255) / 256));
   auto* lat = reinterpret_cast<const __nv_bfloat162*>(latent);
   auto* kp = reinterpret_cast<const __nv_bfloat162*>(k_pe);
   if (c_bits == kC4R4) {

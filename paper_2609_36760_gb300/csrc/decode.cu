@@ -31,7 +31,8 @@
 //                  At a segment end the softmax warps write the final output, or
 //                  an unnormalised partial (m, l, o) when the unit is split.
 //   combine_kernel merges the partials of split units with
-//                  m = max m_j, l = sum e^(m_j - m) l_j, O = sum e^(m_j - m) o_j / l.
+//                  m = max m_j, l = sum e^(m_j - m) l_j, O = sum e^(m_j - m) o_j / l
+//                  (combine_wide_kernel for a few long units).
 #include <cuda_runtime.h>
 
 #include <cstddef>
@@ -1222,8 +1223,11 @@ __global__ void __launch_bounds__(kPrepThreads) prep_kernel(const Params p) {
                         static_cast<int>(idx - static_cast<long long>(u) * kPieces));
     return;
   }
+  constexpr int kSmemUnits = 4096;  // prefixes kept on chip for the per-CTA searches
   __shared__ int warp_sums[32];
   __shared__ int carry;
+  __shared__ int pf_s[kSmemUnits + 1];
+  const bool pf_on_chip = p.batch * p.n_hg < kSmemUnits;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int nwarps = blockDim.x >> 5;
   if (threadIdx.x == 0) carry = 0;
@@ -1260,17 +1264,23 @@ __global__ void __launch_bounds__(kPrepThreads) prep_kernel(const Params p) {
     __syncthreads();
     const int excl = carry + (warp > 0 ? warp_sums[warp - 1] : 0) + x - v;
     if (b < p.batch) {
-      for (int hg = 0; hg < p.n_hg; ++hg) p.prefix_w[b * p.n_hg + hg] = excl + hg * tiles;
+      for (int hg = 0; hg < p.n_hg; ++hg) {
+        p.prefix_w[b * p.n_hg + hg] = excl + hg * tiles;
+        if (pf_on_chip) pf_s[b * p.n_hg + hg] = excl + hg * tiles;
+      }
     }
     __syncthreads();
     if (threadIdx.x == blockDim.x - 1) carry = excl + v;
     __syncthreads();
   }
-  if (threadIdx.x == 0) p.prefix_w[p.batch * p.n_hg] = carry;
+  if (threadIdx.x == 0) {
+    p.prefix_w[p.batch * p.n_hg] = carry;
+    if (pf_on_chip) pf_s[p.batch * p.n_hg] = carry;
+  }
   __syncthreads();
   // The unit holding the first tile of every decode CTA's range (the unit u
   // with prefix[u] <= t0 < prefix[u + 1]), so that no CTA has to search.
-  const volatile int32_t* pf = p.prefix_w;
+  const volatile int32_t* pf = pf_on_chip ? pf_s : p.prefix_w;
   const int units = p.batch * p.n_hg;
   const int T = pf[units];
   for (int c = threadIdx.x; c < p.grid; c += blockDim.x) {
@@ -1356,6 +1366,93 @@ __global__ void __launch_bounds__(128) combine_kernel(const Params p) {
   if (lane == 0 && p.lse != nullptr) p.lse[static_cast<size_t>(b) * p.heads + h0 + h] = (M + log2f(l)) * kLn2;
 }
 
+// The same merge for launches with few units, each split over many CTAs (long
+// contexts): one block per (unit, head) of kWideGroups x 128 threads. Thread i
+// of the first pass holds piece c0 + i's (m, l); block reductions give M and l
+// and the pieces' weights 2^(m_j - M) go to shared memory. Group g then sums
+// pieces c0 + g, c0 + g + kWideGroups, ... for its float4 of every head row,
+// with the loads of several pieces in flight, and the groups' sums are added.
+constexpr int kWideGroups = 4;
+constexpr int kWideThreads = kWideGroups * 128;
+
+template <int HG>
+__global__ void __launch_bounds__(kWideThreads) combine_wide_kernel(const Params p) {
+  __shared__ float red[kWideThreads / 32];
+  __shared__ float wts[kWideThreads];
+  __shared__ float4 part[kWideGroups - 1][128];
+  const int u = blockIdx.x;
+  const int h = blockIdx.y;
+  const int units = p.batch * p.n_hg;
+  const int b = u / p.n_hg;
+  const int h0 = (u - b * p.n_hg) * HG;
+  if (h0 + h >= p.heads) return;
+  const int P0 = p.prefix[u], P1 = p.prefix[u + 1], T = p.prefix[units];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int v = tid & 127, grp = tid >> 7;
+  float4* out = reinterpret_cast<float4*>(p.out + (static_cast<size_t>(b) * p.heads + h0 + h) * kDc) + v;
+  if (P0 == P1) {
+    if (grp == 0) *out = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (p.lse != nullptr && tid == 0) p.lse[static_cast<size_t>(b) * p.heads + h0 + h] = -INFINITY;
+    return;
+  }
+  const int c0 = cta_of(P0, T, p.grid), c1 = cta_of(P1 - 1, T, p.grid);
+  if (c0 == c1) return;  // one CTA covered the whole unit and wrote the result
+  // pieces c0..c1 <= grid <= kWideThreads: one per thread
+  const int c = c0 + tid;
+  float2 ml = make_float2(-INFINITY, 0.0f);
+  if (c <= c1 && p.cta_t0[c] != p.cta_t0[c + 1])  // an empty range wrote no partial
+    ml = __ldcg(reinterpret_cast<const float2*>(p.part_ml) + (static_cast<size_t>(c) + u) * HG + h);
+  float x = ml.x;
+#pragma unroll
+  for (int s = 16; s >= 1; s >>= 1) x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, s));
+  if (lane == 0) red[warp] = x;
+  __syncthreads();
+  float M = red[0];
+#pragma unroll
+  for (int i = 1; i < kWideThreads / 32; ++i) M = fmaxf(M, red[i]);
+  const bool any = M != -INFINITY;  // some piece saw a key
+  const float w = any && ml.x != -INFINITY ? exp2f(ml.x - M) : 0.0f;
+  wts[tid] = w;
+  float y = w * ml.y;
+#pragma unroll
+  for (int s = 16; s >= 1; s >>= 1) y += __shfl_xor_sync(0xffffffffu, y, s);
+  __syncthreads();  // every thread has read red for M
+  if (lane == 0) red[warp] = y;
+  __syncthreads();
+  float L = 0.0f;
+#pragma unroll
+  for (int i = 0; i < kWideThreads / 32; ++i) L += red[i];
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  const float4* ob = reinterpret_cast<const float4*>(p.part_o) + v;
+#pragma unroll 4
+  for (int cc = c0 + grp; cc <= c1; cc += kWideGroups) {
+    const float wc = wts[cc - c0];
+    const float4 o = __ldcg(ob + ((static_cast<size_t>(cc) + u) * HG + h) * (kDc / 4));
+    if (wc != 0.0f) {  // a piece that wrote nothing is never multiplied in
+      acc.x += wc * o.x;
+      acc.y += wc * o.y;
+      acc.z += wc * o.z;
+      acc.w += wc * o.w;
+    }
+  }
+  if (grp > 0) part[grp - 1][v] = acc;
+  __syncthreads();
+  if (grp == 0) {
+#pragma unroll
+    for (int g = 0; g < kWideGroups - 1; ++g) {
+      const float4 q = part[g][v];
+      acc.x += q.x;
+      acc.y += q.y;
+      acc.z += q.z;
+      acc.w += q.w;
+    }
+    const float inv = L > 0.0f ? 1.0f / L : 0.0f;
+    *out = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+    if (tid == 0 && p.lse != nullptr)
+      p.lse[static_cast<size_t>(b) * p.heads + h0 + h] = any ? (M + log2f(L)) * kLn2 : -INFINITY;
+  }
+}
+
 template <int CB, int HG, bool PROT>
 cudaError_t launch_impl(const Params& prm, cudaStream_t stream, cudaEvent_t ev0, cudaEvent_t ev1) {
   static int configured_device = -1;
@@ -1376,7 +1473,13 @@ cudaError_t launch_impl(const Params& prm, cudaStream_t stream, cudaEvent_t ev0,
   decode_main<CB, HG, PROT><<<prm.grid, kThreads, Cfg<HG>::kSmem, stream>>>(prm);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (ev1 != nullptr && (e = cudaEventRecord(ev1, stream)) != cudaSuccess) return e;
-  combine_kernel<HG><<<dim3(static_cast<unsigned>(units), (HG + 3) / 4), 128, 0, stream>>>(prm);
+  // Few units split over many CTAs each (long contexts): spread each unit's
+  // pieces over more threads; otherwise one warp per head.
+  if (units * 4 < prm.grid && prm.grid <= kWideThreads) {
+    combine_wide_kernel<HG><<<dim3(static_cast<unsigned>(units), HG), kWideThreads, 0, stream>>>(prm);
+  } else {
+    combine_kernel<HG><<<dim3(static_cast<unsigned>(units), (HG + 3) / 4), 128, 0, stream>>>(prm);
+  }
   return cudaGetLastError();
 }
 

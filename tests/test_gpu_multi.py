@@ -121,3 +121,13 @@ def test_full_size_dsv3_two_tokens():
     out, lse = c.decode_multi(0, 2)
     assert c.dev_error() == 0
     _check(c, c.lengths_at(0), 0, 2, out, lse, seqs=[0, 31, 63])
+
+
+def test_few_units_with_an_empty_piece():
+    # One sequence of 151 * 128 + 1 tokens: 152 tiles, one per CTA on a 152-SM
+    # GPU, so the last CTA's piece holds only position 19328, which query token 0
+    # may not see. A single unit takes the wide merge, which must skip that piece.
+    c = _case("mq_wide", (151 * 128 + 1,), 16, seed=15)
+    out, lse = c.decode_multi(0, 2, lens=c.prefill)
+    assert c.dev_error() == 0
+    _check(c, c.prefill, 0, 2, out, lse)
