@@ -288,8 +288,13 @@ def run_native(args, ws_world: int, rank: int, local: int):
     if Q.read_dev_err(state.err) != 0:
         raise RuntimeError(f"device error word {Q.read_dev_err(state.err):#x} after warm-up")
 
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
-    for e in ev:
+    # Pass A times whole steps as a user runs them (value); pass B brackets the
+    # main kernel with events (roofline). Events between the library's launches
+    # make each launch wait for the previous one in full, so pass A sets none.
+    Km = min(K, 100)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
+    evm = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(Km)]
+    for e in ev + evm:
         for x in e:
             x.record(stream)
     torch.cuda.synchronize(dev)
@@ -301,14 +306,18 @@ def run_native(args, ws_world: int, rank: int, local: int):
     time.sleep(0.15)
     t_wall0 = time.perf_counter()
     for i in range(K):
-        e0, e1, e_m0, e_m1 = ev[i]
+        e0, e1 = ev[i]
         flush.zero_()
-        Q.set_profile_events(e_m0, e_m1)
         e0.record(stream)
         state.step(Wm + i)
         e1.record(stream)
     torch.cuda.synchronize(dev)
     t_wall = time.perf_counter() - t_wall0
+    for i in range(Km):
+        flush.zero_()
+        Q.set_profile_events(evm[i][0], evm[i][1])
+        state.step(Wm + i)  # the same appends again: the cache is unchanged
+    torch.cuda.synchronize(dev)
     Q.set_profile_events(None, None)
     if dist is not None:
         dist.barrier()
@@ -319,9 +328,9 @@ def run_native(args, ws_world: int, rank: int, local: int):
         raise RuntimeError(f"device error word {err:#x} in the timed loop")
 
     step_ms = [ev[i][0].elapsed_time(ev[i][1]) for i in range(K)]
-    main_ms = [ev[i][2].elapsed_time(ev[i][3]) for i in range(K)]
+    main_ms = [evm[i][0].elapsed_time(evm[i][1]) for i in range(Km)]
     ms_step = sum(step_ms) / K
-    ms_main = sum(main_ms) / K
+    ms_main = sum(main_ms) / Km
     if dist is not None:
         t = torch.tensor([ms_step], device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)

@@ -1184,6 +1184,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   tc_fence_after();
   const uint32_t tmem = ctl.tmem_base;
   if (warp == kMmaWarp && lane != 0) return;  // the MMA role is a single thread
+  // The set-up above may overlap the prep kernel; everything below reads what
+  // prep and the cache writer before it produced.
+  griddep_wait();
 
   Sched sc;
   sc.init(p.prefix, p.cta_info[blockIdx.x], p.batch * p.n_hg, blockIdx.x, gridDim.x);
@@ -1192,6 +1195,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   } else {
     mma_thread<HG>(p, sc, chunks, qsmem, ctl, tmem);
   }
+  griddep_launch_dependents();  // the merge may be scheduled as CTAs finish
   tc_fence_before();
   __syncthreads();  // the exited lanes of the MMA warp do not take part
   if (warp == 0) {
@@ -1212,6 +1216,7 @@ constexpr int kPrepThreads = 1024;
 // Blocks 1..: one query-image piece (16 bytes) per thread.
 template <int CB, int HG>
 __global__ void __launch_bounds__(kPrepThreads) prep_kernel(const Params p) {
+  griddep_launch_dependents();  // the main kernel may start its set-up meanwhile
   if (blockIdx.x > 0) {
     const long long idx = static_cast<long long>(blockIdx.x - 1) * kPrepThreads + threadIdx.x;
     constexpr int kPieces = kNumChunks * HG * 8;
@@ -1303,6 +1308,9 @@ __global__ void __launch_bounds__(kPrepThreads) prep_kernel(const Params p) {
     p.cta_t0[c] = t0;
   }
   if (threadIdx.x == 0) p.cta_t0[p.grid] = T;
+  // prep reads nothing the cache writer before it writes, but the main kernel
+  // waits only for prep: prep does not complete before the writer has.
+  griddep_wait();
 }
 
 // The CTA whose range holds tile t (CTA c's range starts at c * T / grid).
@@ -1317,6 +1325,7 @@ __device__ __forceinline__ int cta_of(int t, int T, int grid) {
 // next partial do not depend on the previous one's arithmetic.
 template <int HG>
 __global__ void __launch_bounds__(128) combine_kernel(const Params p) {
+  griddep_wait();  // the partials of the main kernel
   const int u = blockIdx.x;
   const int h = blockIdx.y * 4 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -1377,6 +1386,7 @@ constexpr int kWideThreads = kWideGroups * 128;
 
 template <int HG>
 __global__ void __launch_bounds__(kWideThreads) combine_wide_kernel(const Params p) {
+  griddep_wait();  // the partials of the main kernel
   __shared__ float red[kWideThreads / 32];
   __shared__ float wts[kWideThreads];
   __shared__ float4 part[kWideGroups - 1][128];
@@ -1453,6 +1463,25 @@ __global__ void __launch_bounds__(kWideThreads) combine_wide_kernel(const Params
   }
 }
 
+// Launches kern on stream; with pdl the launch may overlap the previous kernel
+// in the stream (programmatic stream serialisation), which kern must wait for
+// with griddep_wait before reading its results.
+template <typename... Args>
+cudaError_t launch_k(void (*kern)(Args...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream, bool pdl,
+                     Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 template <int CB, int HG, bool PROT>
 cudaError_t launch_impl(const Params& prm, cudaStream_t stream, cudaEvent_t ev0, cudaEvent_t ev1) {
   static int configured_device = -1;
@@ -1464,23 +1493,27 @@ cudaError_t launch_impl(const Params& prm, cudaStream_t stream, cudaEvent_t ev0,
     if (e != cudaSuccess) return e;
     configured_device = dev;
   }
+  // With measurement events around the main kernel every launch waits for the
+  // previous one in full, so that the events bracket the main kernel alone.
+  const bool pdl = ev0 == nullptr && ev1 == nullptr;
   const long long units = static_cast<long long>(prm.batch) * prm.n_hg;
   const long long pieces = units * kNumChunks * HG * 8;
   const unsigned prep_blocks = static_cast<unsigned>(1 + (pieces + kPrepThreads - 1) / kPrepThreads);
-  prep_kernel<CB, HG><<<prep_blocks, kPrepThreads, 0, stream>>>(prm);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if ((e = launch_k(prep_kernel<CB, HG>, dim3(prep_blocks), dim3(kPrepThreads), 0, stream, pdl, prm)) != cudaSuccess)
+    return e;
   if (ev0 != nullptr && (e = cudaEventRecord(ev0, stream)) != cudaSuccess) return e;
-  decode_main<CB, HG, PROT><<<prm.grid, kThreads, Cfg<HG>::kSmem, stream>>>(prm);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if ((e = launch_k(decode_main<CB, HG, PROT>, dim3(prm.grid), dim3(kThreads), Cfg<HG>::kSmem, stream, pdl, prm)) !=
+      cudaSuccess)
+    return e;
   if (ev1 != nullptr && (e = cudaEventRecord(ev1, stream)) != cudaSuccess) return e;
   // Few units split over many CTAs each (long contexts): spread each unit's
   // pieces over more threads; otherwise one warp per head.
   if (units * 4 < prm.grid && prm.grid <= kWideThreads) {
-    combine_wide_kernel<HG><<<dim3(static_cast<unsigned>(units), HG), kWideThreads, 0, stream>>>(prm);
-  } else {
-    combine_kernel<HG><<<dim3(static_cast<unsigned>(units), (HG + 3) / 4), 128, 0, stream>>>(prm);
+    return launch_k(combine_wide_kernel<HG>, dim3(static_cast<unsigned>(units), HG), dim3(kWideThreads), 0, stream,
+                    pdl, prm);
   }
-  return cudaGetLastError();
+  return launch_k(combine_kernel<HG>, dim3(static_cast<unsigned>(units), (HG + 3) / 4), dim3(128), 0, stream, pdl,
+                  prm);
 }
 
 template <int CB, bool PROT>

@@ -77,6 +77,14 @@ __device__ __forceinline__ int mbar_wait(uint64_t* bar, uint32_t parity, uint64_
   }
 }
 
+// ---------------------------------------------- programmatic dependent launch
+// Wait until the grids this one depends on (launched before it with
+// programmatic stream serialisation) have completed and their memory is
+// visible; a no-op for a grid launched without that attribute.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Allow the next grid in the stream to be scheduled before this one exits.
+__device__ __forceinline__ void griddep_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ----------------------------------------------------- bulk copy (TMA engine)
 // Global -> shared copy of `bytes` (multiple of 16, both addresses 16-byte
 // aligned) completing on `bar` through the transaction count.
