@@ -408,39 +408,67 @@ def cache_name(w: W.Workload, bf16: bool, protect: bool, c4r4: bool) -> str:
 
 def run_e2e(state: Workspace, K: int, flush, dev, tokens: float, n_world: int, dist):
     """Same metric through the public API with the step's inputs in pinned host
-    memory: H2D copies of the appended tokens, queries and lengths, and the D2H
-    read of out and lse, all inside the timed region."""
+    memory: every step copies its appended tokens, queries and lengths host to
+    device and reads out and lse back. The copies are pipelined as a serving loop
+    would run them: step i+1's inputs go in (copy stream) and step i-1's results
+    come out (read-back stream) while step i computes; events order each copy
+    against the step that produces or consumes it. Timed from the first input
+    copy to the last read-back."""
     stream = torch.cuda.current_stream(dev)
-    hs = []
-    for s in range(state.nsteps):
-        h = {k: v.pin_memory() for k, v in state.steps[s]["host"].items()}
-        d = {k: torch.empty_like(v, device=dev) for k, v in h.items()}
-        hs.append((h, d))
-    out_h = torch.empty(state.out.shape, dtype=torch.float32).pin_memory()
-    lse_h = torch.empty(state.lse.shape, dtype=torch.float32).pin_memory()
-    h2d = sum(v.numel() * v.element_size() for v in hs[0][0].values())
-    d2h = out_h.numel() * 4 + lse_h.numel() * 4
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
-    for i in range(K + 3):
-        h, d = hs[i % state.nsteps]
+    h2d_s = torch.cuda.Stream(dev)
+    d2h_s = torch.cuda.Stream(dev)
+    hs = [{k: v.pin_memory() for k, v in state.steps[s]["host"].items()} for s in range(state.nsteps)]
+    dbuf = [{k: torch.empty_like(v, device=dev) for k, v in hs[0].items()} for _ in range(2)]  # inputs of steps i % 2
+    outs = [torch.empty_like(state.out) for _ in range(2)]
+    lses = [torch.empty_like(state.lse) for _ in range(2)]
+    out_h = [torch.empty(state.out.shape, dtype=torch.float32).pin_memory() for _ in range(2)]
+    lse_h = [torch.empty(state.lse.shape, dtype=torch.float32).pin_memory() for _ in range(2)]
+    h2d = sum(v.numel() * v.element_size() for v in hs[0].values())
+    d2h = out_h[0].numel() * 4 + lse_h[0].numel() * 4
+    n = K + 3
+    ev_in = [torch.cuda.Event() for _ in range(n)]
+    ev_done = [torch.cuda.Event() for _ in range(n)]
+    ev_out = [torch.cuda.Event() for _ in range(n)]
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize(dev)
+
+    def issue(i):
+        h, d = hs[i % state.nsteps], dbuf[i % 2]
+        if i >= 2:  # step i - 2 has read this input buffer
+            h2d_s.wait_event(ev_done[i - 2])
+        with torch.cuda.stream(h2d_s):
+            for k in h:
+                d[k].copy_(h[k], non_blocking=True)
+        ev_in[i].record(h2d_s)
+
+    issue(0)
+    for i in range(n):
+        if i + 1 == 3:
+            t0.record(h2d_s)  # the timed steps start with step 3's input copy
+        if i + 1 < n:
+            issue(i + 1)  # the next step's inputs go in while this step computes
+        d = dbuf[i % 2]
+        stream.wait_event(ev_in[i])
+        if i >= 2:
+            stream.wait_event(ev_out[i - 2])  # results buffer i % 2 has been read back
         flush.zero_()
-        if i >= 3:
-            evs[i - 3][0].record(stream)
-        for k in h:
-            d[k].copy_(h[k], non_blocking=True)
-        state.step(i, d)
-        out_h.copy_(state.out, non_blocking=True)
-        lse_h.copy_(state.lse, non_blocking=True)
-        if i >= 3:
-            evs[i - 3][1].record(stream)
-        stream.synchronize()
-    ms = sum(a.elapsed_time(b) for a, b in evs) / K
+        state.step(i, d, out=outs[i % 2], lse=lses[i % 2])
+        ev_done[i].record(stream)
+        d2h_s.wait_event(ev_done[i])
+        with torch.cuda.stream(d2h_s):
+            out_h[i % 2].copy_(outs[i % 2], non_blocking=True)
+            lse_h[i % 2].copy_(lses[i % 2], non_blocking=True)
+        ev_out[i].record(d2h_s)
+    t1.record(d2h_s)
+    torch.cuda.synchronize(dev)
+    ms = t0.elapsed_time(t1) / K
     if dist is not None:
         t = torch.tensor([ms], device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
     return {"value": round(n_world * tokens / (ms * 1e-3), 1), "unit": UNIT, "ms_per_step": round(ms, 5),
-            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": K}
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": K,
+            "pipelined": "step i+1's inputs in and step i-1's results out overlap step i"}
 
 
 # ------------------------------------------------------------------ oracle
