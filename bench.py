@@ -40,7 +40,7 @@ TAU = 1.0 / math.sqrt(192.0)
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
 
 
-def parse():
+def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=2000)
@@ -57,7 +57,7 @@ def parse():
                          "appends that many tokens and scores them under the causal mask")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 def dist_env():
@@ -65,6 +65,22 @@ def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     return ws, rank, local
+
+
+def max_over_ranks(x: float, dist, device) -> float:
+    """The largest x over all ranks (x itself without a process group): the job's
+    time is its slowest rank's."""
+    if dist is None:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_value(world: int, tokens_per_rank_step: float, ms_per_step: float) -> float:
+    """KV tokens per second over all ranks: every rank decodes its own replica of
+    the workload in the same (slowest-rank) step time."""
+    return world * tokens_per_rank_step / (ms_per_step * 1e-3)
 
 
 def load_peaks():
@@ -331,16 +347,11 @@ def run_native(args, ws_world: int, rank: int, local: int):
     main_ms = [evm[i][0].elapsed_time(evm[i][1]) for i in range(Km)]
     ms_step = sum(step_ms) / K
     ms_main = sum(main_ms) / Km
-    if dist is not None:
-        t = torch.tensor([ms_step], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_step_max = float(t.item())
-    else:
-        ms_step_max = ms_step
+    ms_step_max = max_over_ranks(ms_step, dist, dev)
 
     lens_all = [state.steps[(Wm + i) % state.nsteps]["lens"] for i in range(K)]
     tok_per_step = sum(sum(l) for l in lens_all) / K
-    value = ws_world * tok_per_step / (ms_step_max * 1e-3)
+    value = whole_job_value(ws_world, tok_per_step, ms_step_max)
 
     # roofline of the main decode kernel
     peaks, peak_src = load_peaks()
@@ -461,12 +472,8 @@ def run_e2e(state: Workspace, K: int, flush, dev, tokens: float, n_world: int, d
         ev_out[i].record(d2h_s)
     t1.record(d2h_s)
     torch.cuda.synchronize(dev)
-    ms = t0.elapsed_time(t1) / K
-    if dist is not None:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    return {"value": round(n_world * tokens / (ms * 1e-3), 1), "unit": UNIT, "ms_per_step": round(ms, 5),
+    ms = max_over_ranks(t0.elapsed_time(t1) / K, dist, dev)
+    return {"value": round(whole_job_value(n_world, tokens, ms), 1), "unit": UNIT, "ms_per_step": round(ms, 5),
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "steps": K,
             "pipelined": "step i+1's inputs in and step i-1's results out overlap step i"}
 
