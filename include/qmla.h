@@ -321,6 +321,27 @@ int qmla_mla_decode_static(const void* pool_dev, int c_bits, int num_blocks, con
                            int max_blocks, const int32_t* seq_lens_dev, float softmax_scale, float* out_dev,
                            float* lse_dev, uint32_t* dev_err_dev, qmla_stream_t stream);
 
+/*
+ * Test hook (no counterpart in the paper): the fp16 tile the decode kernel builds
+ * from the cache for tile j (positions 128 j .. 128 j + 127) of sequence b, made
+ * by the decode's own row loaders into its swizzled shared-memory chunks and
+ * written out row-major in channel order.
+ *   cache_kind   4 or 2: this library's block with that content width;
+ *                QMLA_CACHE_C4R4: the paper's page; QMLA_CACHE_BF16: the BF16 cache
+ *   prot_dev     NULL, or the sink4/local128 protection buffer (packed kinds):
+ *                rows in P_L come from it as in qmla_mla_decode_protected
+ *   tile_dev     [128][576] fp16 (uint16 bits), 16-byte aligned; row r holds the
+ *                512 latent then 64 RoPE-key values of position 128 j + r, zero for
+ *                rows at or past seq_lens_dev[b]
+ * Table, lengths and errors as qmla_mla_decode; 0 <= b < batch, 0 <= j. One CTA
+ * of 128 threads; not a fast path.
+ */
+#define QMLA_CACHE_C4R4 5
+#define QMLA_CACHE_BF16 16
+int qmla_debug_tile(const void* pool_dev, int cache_kind, int num_blocks, const int32_t* block_table_dev,
+                    int max_blocks, const int32_t* seq_lens_dev, int batch, int b, int j, const void* prot_dev,
+                    uint16_t* tile_dev, uint32_t* dev_err_dev, qmla_stream_t stream);
+
 /* Copies the device error word to *host_out after synchronising `stream`. */
 int qmla_read_dev_err(const uint32_t* dev_err_dev, uint32_t* host_out, qmla_stream_t stream);
 

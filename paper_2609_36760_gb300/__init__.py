@@ -76,6 +76,8 @@ def lib():
     L.qmla_mla_decode_multi.argtypes = [vp, i32, i32, vp, vp, i32, i32, i32, vp, i32, vp, vp, f32, vp, vp, vp, sz,
                                         vp, vp]
     L.qmla_mla_decode_multi.restype = i32
+    L.qmla_debug_tile.argtypes = [vp, i32, i32, vp, i32, vp, i32, i32, i32, vp, vp, vp, vp]
+    L.qmla_debug_tile.restype = i32
     L.qmla_c4r4_page_bytes.argtypes, L.qmla_c4r4_page_bytes.restype = [], sz
     L.qmla_quant_append_c4r4.argtypes = [vp, i32, vp, vp, vp, vp, i32, vp, i32, i32, vp, vp, vp, vp]
     L.qmla_quant_append_c4r4.restype = i32
@@ -196,6 +198,21 @@ def mla_decode_multi(pool: torch.Tensor, c_bits: int, q_latent: torch.Tensor, q_
                                      float(softmax_scale), _ptr(out), _ptr(lse), _ptr(workspace),
                                      workspace.numel() * workspace.element_size(), _ptr(dev_err), _stream(stream))
     _check("qmla_mla_decode_multi", st)
+
+
+CACHE_C4R4 = 5   # qmla_debug_tile cache kinds (besides content bit widths 4 and 2)
+CACHE_BF16 = 16
+
+
+def debug_tile(pool: torch.Tensor, cache_kind: int, block_table: torch.Tensor, seq_lens: torch.Tensor, b: int,
+               j: int, tile: torch.Tensor, dev_err: torch.Tensor, prot: torch.Tensor | None = None,
+               stream=None) -> None:
+    """qmla_debug_tile: tile j of sequence b as the decode kernel builds it, into
+    tile [128, 576] (fp16 or int16)."""
+    st = lib().qmla_debug_tile(_ptr(pool), cache_kind, pool.shape[0], _ptr(block_table), block_table.shape[1],
+                               _ptr(seq_lens), block_table.shape[0], b, j, _ptr(prot), _ptr(tile), _ptr(dev_err),
+                               _stream(stream))
+    _check("qmla_debug_tile", st)
 
 
 def c4r4_page_bytes() -> int:

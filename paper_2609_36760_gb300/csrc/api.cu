@@ -263,6 +263,37 @@ int qmla_mla_decode_bf16cache(const void* pool_dev, int num_blocks, const uint16
                        stream);
 }
 
+int qmla_debug_tile(const void* pool_dev, int cache_kind, int num_blocks, const int32_t* block_table_dev,
+                    int max_blocks, const int32_t* seq_lens_dev, int batch, int b, int j, const void* prot_dev,
+                    uint16_t* tile_dev, uint32_t* dev_err_dev, qmla_stream_t stream) {
+  static_assert(QMLA_CACHE_C4R4 == qmla::kC4R4, "kind code of the paper's page");
+  if (cache_kind != 4 && cache_kind != 2 && cache_kind != QMLA_CACHE_C4R4 && cache_kind != QMLA_CACHE_BF16)
+    return QMLA_ERR_INVALID_ARG;
+  if (pool_dev == nullptr || block_table_dev == nullptr || seq_lens_dev == nullptr || tile_dev == nullptr)
+    return QMLA_ERR_INVALID_ARG;
+  if (num_blocks <= 0 || max_blocks <= 0 || batch <= 0 || b < 0 || b >= batch || j < 0 ||
+      static_cast<long long>(j) * 2 >= max_blocks)
+    return QMLA_ERR_INVALID_ARG;
+  if (!aligned(pool_dev, 16) || !aligned(tile_dev, 16) || (prot_dev != nullptr && !aligned(prot_dev, 16)))
+    return QMLA_ERR_INVALID_ARG;
+  if (prot_dev != nullptr && cache_kind == QMLA_CACHE_BF16) return QMLA_ERR_INVALID_ARG;
+  DevInfo di;
+  int st = current_device_info(di);
+  if (st != QMLA_OK) return st;
+  qmla::DecodeArgs a;
+  a.pool = pool_dev;
+  a.cache_kind = cache_kind;
+  a.num_blocks = num_blocks;
+  a.batch = batch;
+  a.table = block_table_dev;
+  a.max_blocks = max_blocks;
+  a.seq_lens = seq_lens_dev;
+  a.dev_err = dev_err_dev;
+  a.prot = prot_dev;
+  cudaError_t e = qmla::launch_tile_dump(a, b, j, tile_dev, reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
+}
+
 int qmla_read_dev_err(const uint32_t* dev_err_dev, uint32_t* host_out, qmla_stream_t stream) {
   if (dev_err_dev == nullptr || host_out == nullptr) return QMLA_ERR_INVALID_ARG;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

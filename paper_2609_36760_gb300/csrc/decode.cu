@@ -784,6 +784,29 @@ __device__ bool epilogue(const Params& p, const SegEnd& e, Ctrl& ctl, uint32_t t
   return true;
 }
 
+// Chunk k of one tile row of a packed cache: the protected bf16 row when ps is
+// set, else the packed row f dequantised (the paper's page or this library's
+// block). The decode workers and the tile dump share it.
+template <int CB, bool PROT>
+__device__ __forceinline__ void dq_row(uint32_t chunk_base, int row, int k, const uint8_t* ps, const Fetch& f) {
+  if (PROT && ps != nullptr) {
+    uint4 pv[8];  // the protected row's 64 bf16 values of chunk k
+    // L1-allocating loads: the eight 16-byte pieces of the row's 128-byte line
+    // come from one L1 fill instead of eight L2 reads.
+#pragma unroll
+    for (int i = 0; i < 8; ++i) pv[i] = __ldg(reinterpret_cast<const uint4*>(ps + k * 128) + i);
+    store_row_prot<CB>(chunk_base, row, pv, k);
+  } else if constexpr (CB == kC4R4) {
+    if (k < 8) {
+      store_row_c4r4<true>(chunk_base, row, f);
+    } else {
+      store_row_c4r4<false>(chunk_base, row, f);
+    }
+  } else {
+    store_row<CB>(chunk_base, row, f, CB == 4 || k == 8);
+  }
+}
+
 // PROT: the cache has sink4/local128 protection rows (a separate instantiation,
 // so the unprotected kernel carries none of that code).
 template <int CB, int HG, bool PROT>
@@ -894,24 +917,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
 #pragma unroll
         for (int i = 0; i < 8; ++i) cur[i] = nxt[i];
       } else {
-        if (PROT && psrc_cur != nullptr) {
-          uint4 pv[8];  // the protected row's 64 bf16 values of chunk k
-#pragma unroll
-          // L1-allocating loads: the eight 16-byte pieces of the row's 128-byte
-          // line come from one L1 fill instead of eight L2 reads.
-          for (int i = 0; i < 8; ++i) pv[i] = __ldg(reinterpret_cast<const uint4*>(psrc_cur + k * 128) + i);
-          store_row_prot<CB>(chunks + k * kChunkBytes, row, pv, k);
-        } else {
-          if constexpr (CB == kC4R4) {
-            if (k < 8) {
-              store_row_c4r4<true>(chunks + k * kChunkBytes, row, f[kc]);
-            } else {
-              store_row_c4r4<false>(chunks + k * kChunkBytes, row, f[kc]);
-            }
-          } else {
-            store_row<CB>(chunks + k * kChunkBytes, row, f[kc], CB == 4 || k == 8);
-          }
-        }
+        dq_row<CB, PROT>(chunks + k * kChunkBytes, row, k, psrc_cur, f[kc]);
         f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);  // the next tile's rows of this chunk
       }
       fence_proxy_async_smem();
@@ -1463,6 +1469,69 @@ __global__ void __launch_bounds__(kWideThreads) combine_wide_kernel(const Params
   }
 }
 
+// Test hook: the fp16 tile the decode kernel builds for tile j (tokens 128 j ..
+// 128 j + 127) of sequence b, made by the same row loaders (packed rows
+// dequantised, protected rows and BF16 rows converted) into the same swizzled
+// chunks, then written out row-major in channel order: out [128][576] fp16,
+// rows past the sequence end zero.
+template <int CB, bool PROT>
+__global__ void __launch_bounds__(kTileTokens) tile_dump_kernel(const Params p, int b, int j, uint16_t* out) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const uint32_t chunks = smem_u32(smem);
+  const int row = threadIdx.x;
+  const int slot = row & 63;
+  RowRef r;
+  r.has = true;
+  r.b = b;
+  r.j = j;
+  r.len = p.seq_lens[b];
+  r.entry = p.table[static_cast<size_t>(b) * p.max_blocks + min(2 * j + (row >= 64 ? 1 : 0), p.max_blocks - 1)];
+  bool valid = false;
+  const uint8_t* ps = PROT ? prot_row(p, r, row) : nullptr;
+  const uint8_t* blk = resolve_row<CB>(p, r, row, valid);
+#pragma unroll 1
+  for (int k = 0; k < kNumChunks; ++k) {
+    const uint32_t cbase = chunks + k * kChunkBytes;
+    if constexpr (CB == 16) {
+      uint4 v[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+        v[i] = valid ? ldg_nc_v4(blk + slot * (kDqk * 2) + k * 128 + i * 16) : make_uint4(0, 0, 0, 0);
+      store_row_bf16(cbase, row, v, valid);
+    } else {
+      const Fetch f = fetch_chunk<CB>(blk, valid && ps == nullptr, k, slot);
+      dq_row<CB, PROT>(cbase, row, k, ps, f);
+    }
+  }
+  __syncthreads();
+#pragma unroll 1
+  for (int k = 0; k < kNumChunks; ++k) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      uint32_t w[4];
+      asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];"
+                   : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3])
+                   : "r"(chunks + k * kChunkBytes + swz_off(row, i, 128)));
+      const uint16_t* h = reinterpret_cast<const uint16_t*>(w);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const int ch = CB == 16 ? e : (k == 8 ? Perm<4>::at(e) : Perm<CB>::at(e));
+        out[static_cast<size_t>(row) * kDqk + k * 64 + i * 8 + ch] = h[e];
+      }
+    }
+  }
+}
+
+template <int CB, bool PROT>
+cudaError_t launch_tile_dump(const Params& prm, int b, int j, uint16_t* out, cudaStream_t stream) {
+  constexpr int kSmem = 1024 + kNumChunks * kChunkBytes;
+  cudaError_t e = cudaFuncSetAttribute(tile_dump_kernel<CB, PROT>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+  if (e != cudaSuccess) return e;
+  tile_dump_kernel<CB, PROT><<<1, kTileTokens, kSmem, stream>>>(prm, b, j, out);
+  return cudaGetLastError();
+}
+
 // Launches kern on stream; with pdl the launch may overlap the previous kernel
 // in the stream (programmatic stream serialisation), which kern must wait for
 // with griddep_wait before reading its results.
@@ -1595,7 +1664,29 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
   return launch_hg<16, false>(hg, prm, stream, a.ev_before_main, a.ev_after_main);
 }
 
+cudaError_t launch_tile_dump(const DecodeArgs& a, int b, int j, uint16_t* out, cudaStream_t stream) {
+  Params prm{};
+  prm.pool = static_cast<const uint8_t*>(a.pool);
+  prm.prot = a.cache_kind == 16 ? nullptr : static_cast<const uint8_t*>(a.prot);
+  prm.num_blocks = a.num_blocks;
+  prm.batch = a.batch;
+  prm.table = a.table;
+  prm.max_blocks = a.max_blocks;
+  prm.seq_lens = a.seq_lens;
+  prm.dev_err = a.dev_err;
+  const bool prot = prm.prot != nullptr;
+  switch (a.cache_kind) {
+    case 4: return prot ? launch_tile_dump<4, true>(prm, b, j, out, stream) : launch_tile_dump<4, false>(prm, b, j, out, stream);
+    case 2: return prot ? launch_tile_dump<2, true>(prm, b, j, out, stream) : launch_tile_dump<2, false>(prm, b, j, out, stream);
+    case kC4R4:
+      return prot ? launch_tile_dump<kC4R4, true>(prm, b, j, out, stream)
+                  : launch_tile_dump<kC4R4, false>(prm, b, j, out, stream);
+    default: return launch_tile_dump<16, false>(prm, b, j, out, stream);
+  }
+}
+
 #ifdef QMLA_TRACE_BUILD
+cudaError_t set_trace_buffer(void* buf) {#ifdef QMLA_TRACE_BUILD
 cudaError_t set_trace_buffer(void* buf) {
   g_trace_buf = static_cast<unsigned long long*>(buf);
   return cudaSuccess;

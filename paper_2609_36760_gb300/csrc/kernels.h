@@ -49,6 +49,8 @@ struct DecodeArgs {
   cudaEvent_t ev_after_main = nullptr;
 };
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
+// Test hook: tile j of sequence b as the decode kernel builds it, [128][576] fp16.
+cudaError_t launch_tile_dump(const DecodeArgs& a, int b, int j, uint16_t* out, cudaStream_t stream);
 
 // Records a failed CUDA call for qmla_last_cuda_error (calling thread).
 void record_cuda_error(int err);
