@@ -342,6 +342,15 @@ int qmla_debug_tile(const void* pool_dev, int cache_kind, int num_blocks, const 
                     int max_blocks, const int32_t* seq_lens_dev, int batch, int b, int j, const void* prot_dev,
                     uint16_t* tile_dev, uint32_t* dev_err_dev, qmla_stream_t stream);
 
+/* Test hook (no counterpart in the paper): one warp waits, through the decode
+ * kernel's bounded wait, for a barrier phase that nothing completes. After
+ * limit_us microseconds (1 .. 1000000) the wait gives up and ORs
+ * QMLA_DEVERR_TIMEOUT | QMLA_DEVERR_SITE_SOFTMAX into *dev_err_dev, and the
+ * kernel returns; the context stays usable. The decode's own waits give up after
+ * 2 s the same way (one site bit per wait, bits 8 and up). */
+#define QMLA_DEVERR_SITE_SOFTMAX (0x100u << 5)
+int qmla_debug_wait_timeout(uint32_t limit_us, uint32_t* dev_err_dev, qmla_stream_t stream);
+
 /* Copies the device error word to *host_out after synchronising `stream`. */
 int qmla_read_dev_err(const uint32_t* dev_err_dev, uint32_t* host_out, qmla_stream_t stream);
 

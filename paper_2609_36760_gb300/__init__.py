@@ -76,6 +76,8 @@ def lib():
     L.qmla_mla_decode_multi.argtypes = [vp, i32, i32, vp, vp, i32, i32, i32, vp, i32, vp, vp, f32, vp, vp, vp, sz,
                                         vp, vp]
     L.qmla_mla_decode_multi.restype = i32
+    L.qmla_debug_wait_timeout.argtypes = [ctypes.c_uint32, vp, vp]
+    L.qmla_debug_wait_timeout.restype = i32
     L.qmla_debug_tile.argtypes = [vp, i32, i32, vp, i32, vp, i32, i32, i32, vp, vp, vp, vp]
     L.qmla_debug_tile.restype = i32
     L.qmla_c4r4_page_bytes.argtypes, L.qmla_c4r4_page_bytes.restype = [], sz
@@ -213,6 +215,14 @@ def debug_tile(pool: torch.Tensor, cache_kind: int, block_table: torch.Tensor, s
                                _ptr(seq_lens), block_table.shape[0], b, j, _ptr(prot), _ptr(tile), _ptr(dev_err),
                                _stream(stream))
     _check("qmla_debug_tile", st)
+
+
+DEVERR_SITE_SOFTMAX = 0x100 << 5
+
+
+def debug_wait_timeout(limit_us: int, dev_err: torch.Tensor, stream=None) -> None:
+    """qmla_debug_wait_timeout: a decode wait that runs out after limit_us."""
+    _check("qmla_debug_wait_timeout", lib().qmla_debug_wait_timeout(limit_us, _ptr(dev_err), _stream(stream)))
 
 
 def c4r4_page_bytes() -> int:

@@ -294,6 +294,16 @@ int qmla_debug_tile(const void* pool_dev, int cache_kind, int num_blocks, const 
   return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
 }
 
+int qmla_debug_wait_timeout(uint32_t limit_us, uint32_t* dev_err_dev, qmla_stream_t stream) {
+  if (dev_err_dev == nullptr || limit_us < 1u || limit_us > 1000000u) return QMLA_ERR_INVALID_ARG;
+  DevInfo di;
+  int st = current_device_info(di);
+  if (st != QMLA_OK) return st;
+  cudaError_t e = qmla::launch_wait_timeout(dev_err_dev, static_cast<unsigned long long>(limit_us) * 1000ull,
+                                            reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
+}
+
 int qmla_read_dev_err(const uint32_t* dev_err_dev, uint32_t* host_out, qmla_stream_t stream) {
   if (dev_err_dev == nullptr || host_out == nullptr) return QMLA_ERR_INVALID_ARG;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

@@ -240,8 +240,8 @@ __device__ __forceinline__ bool wait_ok(int r, uint32_t site, Ctrl& c, uint32_t*
 // of other warps' shared-memory stores by thousands of cycles, and its own
 // wake-up after the phase completed took ~2k cycles.
 __device__ __forceinline__ bool wwait(uint64_t* bar, uint32_t parity, Ctrl& c, uint32_t site,
-                                      uint32_t* dev_err) {
-  const int r = mbar_wait(bar, parity, kWaitNs, &c.abort);
+                                      uint32_t* dev_err, uint64_t limit_ns = kWaitNs) {
+  const int r = mbar_wait(bar, parity, limit_ns, &c.abort);
   const bool all_ok = __all_sync(0xffffffffu, r == 1);
   if (r == 0) wait_ok(r, site, c, dev_err);
   return all_ok;
@@ -1532,6 +1532,20 @@ cudaError_t launch_tile_dump(const Params& prm, int b, int j, uint16_t* out, cud
   return cudaGetLastError();
 }
 
+// Test hook: one warp waits, through the decode's own bounded wait, for a
+// barrier phase that nothing completes; after limit_ns it reports
+// QMLA_DEVERR_TIMEOUT and the wait site's bit in the error word and returns.
+__global__ void __launch_bounds__(32) wait_timeout_kernel(uint32_t* dev_err, unsigned long long limit_ns) {
+  __shared__ Ctrl ctl;
+  if (threadIdx.x == 0) {
+    mbar_init(&ctl.s_full, 1);  // never arrived on
+    ctl.abort = 0u;
+    fence_mbar_init();
+  }
+  __syncwarp();
+  (void)wwait(&ctl.s_full, 0u, ctl, kSiteSmSFull, dev_err, limit_ns);
+}
+
 // Launches kern on stream; with pdl the launch may overlap the previous kernel
 // in the stream (programmatic stream serialisation), which kern must wait for
 // with griddep_wait before reading its results.
@@ -1685,8 +1699,12 @@ cudaError_t launch_tile_dump(const DecodeArgs& a, int b, int j, uint16_t* out, c
   }
 }
 
+cudaError_t launch_wait_timeout(uint32_t* dev_err, unsigned long long limit_ns, cudaStream_t stream) {
+  wait_timeout_kernel<<<1, 32, 0, stream>>>(dev_err, limit_ns);
+  return cudaGetLastError();
+}
+
 #ifdef QMLA_TRACE_BUILD
-cudaError_t set_trace_buffer(void* buf) {#ifdef QMLA_TRACE_BUILD
 cudaError_t set_trace_buffer(void* buf) {
   g_trace_buf = static_cast<unsigned long long*>(buf);
   return cudaSuccess;

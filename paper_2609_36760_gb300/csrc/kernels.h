@@ -51,6 +51,8 @@ struct DecodeArgs {
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
 // Test hook: tile j of sequence b as the decode kernel builds it, [128][576] fp16.
 cudaError_t launch_tile_dump(const DecodeArgs& a, int b, int j, uint16_t* out, cudaStream_t stream);
+// Test hook: a decode wait that runs out after limit_ns (see qmla_debug_wait_timeout).
+cudaError_t launch_wait_timeout(uint32_t* dev_err, unsigned long long limit_ns, cudaStream_t stream);
 
 // Records a failed CUDA call for qmla_last_cuda_error (calling thread).
 void record_cuda_error(int err);

@@ -105,3 +105,15 @@ def test_multi_query_host_checks(libqmla):
     args = list(base)
     args[11] = ctypes.c_void_p(0x10008)                          # misaligned protection buffer
     assert L.qmla_mla_decode_multi(*args) == 1
+
+
+def test_debug_hooks_host_checks(libqmla):
+    L = libqmla
+    fake = ctypes.c_void_p(0x10000)
+    assert L.qmla_debug_wait_timeout(0, fake, None) == 1          # limit below 1 us
+    assert L.qmla_debug_wait_timeout(1000001, fake, None) == 1    # above 1 s
+    assert L.qmla_debug_wait_timeout(10, None, None) == 1         # no error word
+    # tile dump: bad kind, sequence outside the batch, tile beyond the table
+    assert L.qmla_debug_tile(fake, 3, 4, fake, 2, fake, 1, 0, 0, None, fake, None, None) == 1
+    assert L.qmla_debug_tile(fake, 4, 4, fake, 2, fake, 1, 1, 0, None, fake, None, None) == 1
+    assert L.qmla_debug_tile(fake, 4, 4, fake, 2, fake, 1, 0, 1, None, fake, None, None) == 1
