@@ -117,3 +117,14 @@ def test_debug_hooks_host_checks(libqmla):
     assert L.qmla_debug_tile(fake, 3, 4, fake, 2, fake, 1, 0, 0, None, fake, None, None) == 1
     assert L.qmla_debug_tile(fake, 4, 4, fake, 2, fake, 1, 1, 0, None, fake, None, None) == 1
     assert L.qmla_debug_tile(fake, 4, 4, fake, 2, fake, 1, 0, 1, None, fake, None, None) == 1
+
+
+def test_trace_build_compiles(tmp_path):
+    # The event-timeline variant of the decode (-DQMLA_TRACE_BUILD) is a separate
+    # preprocessor path; compile it so it cannot rot unnoticed.
+    import subprocess
+    from paper_2609_36760_gb300 import build
+    src = os.path.join(build.CSRC, "decode.cu")
+    cmd = [build.nvcc(), *build.ARCH, *build.FLAGS, "-DQMLA_TRACE_BUILD", "-c", src, "-o", str(tmp_path / "d.o")]
+    res = subprocess.run(cmd, stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True)
+    assert res.returncode == 0, res.stdout[-2000:]
