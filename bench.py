@@ -260,6 +260,9 @@ class Workspace:
         out = self.out if out is None else out
         lse = self.lse if lse is None else lse
         self._append(d["lat"], d["kp"], d["sid"], d["pos"], d["lens"])
+        self.decode(d, out, lse)
+
+    def decode(self, d: dict, out, lse):
         if self.q_tokens > 1:
             self.Q.mla_decode_multi(self.pool, self.w.c_bits, d["ql"], d["qp"], self.table, d["lens"], TAU, out,
                                     lse, self.ws, self.err, prot=self.prot)
@@ -309,7 +312,8 @@ def run_native(args, ws_world: int, rank: int, local: int):
     # make each launch wait for the previous one in full, so pass A sets none.
     Km = min(K, 100)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
-    evm = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(Km)]
+    # pass B events: before the append, after it, around the main kernel (set in the library), after the merge
+    evm = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(Km)]
     for e in ev + evm:
         for x in e:
             x.record(stream)
@@ -330,9 +334,15 @@ def run_native(args, ws_world: int, rank: int, local: int):
     torch.cuda.synchronize(dev)
     t_wall = time.perf_counter() - t_wall0
     for i in range(Km):
+        a0, a1, m0, m1, e_end = evm[i]
         flush.zero_()
-        Q.set_profile_events(evm[i][0], evm[i][1])
-        state.step(Wm + i)  # the same appends again: the cache is unchanged
+        Q.set_profile_events(m0, m1)
+        d = state.steps[(Wm + i) % state.nsteps]["dev"]
+        a0.record(stream)
+        state._append(d["lat"], d["kp"], d["sid"], d["pos"], d["lens"])  # the same appends again: cache unchanged
+        a1.record(stream)
+        state.decode(d, state.out, state.lse)
+        e_end.record(stream)
     torch.cuda.synchronize(dev)
     Q.set_profile_events(None, None)
     if dist is not None:
@@ -344,7 +354,15 @@ def run_native(args, ws_world: int, rank: int, local: int):
         raise RuntimeError(f"device error word {err:#x} in the timed loop")
 
     step_ms = [ev[i][0].elapsed_time(ev[i][1]) for i in range(K)]
-    main_ms = [evm[i][0].elapsed_time(evm[i][1]) for i in range(Km)]
+    main_ms = [evm[i][2].elapsed_time(evm[i][3]) for i in range(Km)]
+    med = lambda xs: statistics.median(xs) * 1e3  # noqa: E731
+    parts_us = {"append": round(med([e[0].elapsed_time(e[1]) for e in evm]), 2),
+                "prep_and_gaps": round(med([e[1].elapsed_time(e[2]) for e in evm]), 2),
+                "main": round(med(main_ms), 2),
+                "merge_and_gap": round(med([e[3].elapsed_time(e[4]) for e in evm]), 2),
+                "note": "medians of pass B, whose events serialise the launches"}
+    qs = statistics.quantiles(step_ms, n=10) if K >= 10 else [min(step_ms)] * 9
+    step_dist_us = {"median": round(med(step_ms), 2), "p10": round(qs[0] * 1e3, 2), "p90": round(qs[-1] * 1e3, 2)}
     ms_step = sum(step_ms) / K
     ms_main = sum(main_ms) / Km
     ms_step_max = max_over_ranks(ms_step, dist, dev)
@@ -394,6 +412,8 @@ def run_native(args, ws_world: int, rank: int, local: int):
                    "kv_tokens_per_step_per_gpu": tok_per_step, "l2": "flushed (256 MB write) before every timed step",
                    "parallelism": f"replicas x{ws_world} (independent sequences)"},
         "us_per_step": round(ms_step_max * 1e3, 2),
+        "us_per_step_dist": step_dist_us,
+        "step_parts_us": parts_us,
         "roofline": roof,
         "gpu_launches": state.launches_per_step() * K,
         "clocks": clk,
