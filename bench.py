@@ -55,6 +55,9 @@ def parse(argv=None):
     ap.add_argument("--q-tokens", type=int, default=1,
                     help="query tokens per sequence (multi-token prediction / speculative verification); each step "
                          "appends that many tokens and scores them under the causal mask")
+    ap.add_argument("--pair", action="store_true",
+                    help="decode on CTA pairs (qmla_mla_decode_pair; heads x q-tokens a multiple of 128, "
+                         "INT4/INT2 block, no protection)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args(argv)
@@ -182,10 +185,13 @@ class Workspace:
     """GPU state of one workload: pool, block table, per-step inputs."""
 
     def __init__(self, w: W.Workload, bf16: bool, dev: torch.device, nsteps: int, protect: bool = False,
-                 c4r4: bool = False, q_tokens: int = 1):
+                 c4r4: bool = False, q_tokens: int = 1, pair: bool = False):
         import paper_2609_36760_gb300 as Q
         self.Q = Q
         self.q_tokens = q_tokens
+        self.pair = pair
+        if pair and (bf16 or c4r4 or protect or (q_tokens * w.heads) % 128 != 0):
+            raise SystemExit("--pair decodes the INT4/INT2 block without protection, heads x q-tokens % 128 == 0")
         if q_tokens > 1:
             if bf16 or c4r4:
                 raise SystemExit("--q-tokens > 1 runs on the INT4/INT2 block (protection optional)")
@@ -263,7 +269,10 @@ class Workspace:
         self.decode(d, out, lse)
 
     def decode(self, d: dict, out, lse):
-        if self.q_tokens > 1:
+        if self.pair:
+            self.Q.mla_decode_pair(self.pool, self.w.c_bits, d["ql"], d["qp"], self.table, d["lens"], TAU, out, lse,
+                                   self.ws, self.err)
+        elif self.q_tokens > 1:
             self.Q.mla_decode_multi(self.pool, self.w.c_bits, d["ql"], d["qp"], self.table, d["lens"], TAU, out,
                                     lse, self.ws, self.err, prot=self.prot)
         elif self.c4r4:
@@ -294,7 +303,8 @@ def run_native(args, ws_world: int, rank: int, local: int):
         dist.init_process_group("nccl", device_id=dev)
     w = W.WORKLOADS[args.workload]
     K, Wm = args.steps, args.warmup
-    state = Workspace(w, args.bf16_cache, dev, K + Wm, protect=args.protect, c4r4=args.c4r4, q_tokens=args.q_tokens)
+    state = Workspace(w, args.bf16_cache, dev, K + Wm, protect=args.protect, c4r4=args.c4r4, q_tokens=args.q_tokens,
+                      pair=args.pair)
     w = state.w
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # larger than the 126 MB L2
     stream = torch.cuda.current_stream(dev)
@@ -390,8 +400,9 @@ def run_native(args, ws_world: int, rank: int, local: int):
                        and bool(prof.get("bf16_cache")) == bool(args.bf16_cache)
                        and bool(prof.get("protect")) == bool(args.protect)
                        and bool(prof.get("c4r4")) == bool(state.c4r4)
-                       and int(prof.get("q_tokens", 1)) == args.q_tokens else None)
-    roof["kernel"] = "decode_main"
+                       and int(prof.get("q_tokens", 1)) == args.q_tokens
+                       and bool(prof.get("pair")) == bool(args.pair) else None)
+    roof["kernel"] = "decode_pair" if args.pair else "decode_main"
     roof["kernel_us"] = round(ms_main * 1e3, 2)
     roof["algorithmic_flops"] = flops
     roof["algorithmic_bytes"] = nbytes
@@ -409,6 +420,7 @@ def run_native(args, ws_world: int, rank: int, local: int):
         "config": {"workload": w.name, "batch_per_gpu": w.batch, "heads": w.heads, "c_bits": w.c_bits,
                    "pe_bits": 4, "cache": cache_name(w, args.bf16_cache, args.protect, state.c4r4),
                    "q_tokens_per_seq": args.q_tokens,
+                   "kernel": "CTA pairs (qmla_mla_decode_pair)" if args.pair else "one CTA per SM (qmla_mla_decode)",
                    "kv_tokens_per_step_per_gpu": tok_per_step, "l2": "flushed (256 MB write) before every timed step",
                    "parallelism": f"replicas x{ws_world} (independent sequences)"},
         "us_per_step": round(ms_step_max * 1e3, 2),

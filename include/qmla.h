@@ -229,6 +229,23 @@ int qmla_mla_decode_multi(const void* pool_dev, int c_bits, int num_blocks, cons
                           void* workspace_dev, size_t workspace_bytes, uint32_t* dev_err_dev,
                           qmla_stream_t stream);
 
+/* qmla_mla_decode_multi (INT4 / INT2 block, no protection) on pairs of CTAs
+ * (thread-block clusters of two): each unit of 128 query rows of a sequence is
+ * computed by two SMs, each holding half of the 576 channels of every
+ * reconstructed tile and the matching half of the output; the partial scores
+ * and the softmax weights P of Eq. mla_compact are exchanged between the two
+ * through distributed shared memory, so every MMA spans all 128 query rows
+ * (App. C.5 "cache update and tile reuse"; the split results are merged with
+ * the "global attention normalization" rule as in qmla_mla_decode).
+ * q_tokens x heads must be a multiple of 128 (QMLA_ERR_UNSUPPORTED otherwise);
+ * layouts, workspace size (qmla_decode_workspace_bytes(batch, q_tokens *
+ * heads)), results and errors as qmla_mla_decode_multi with prot_dev = NULL. */
+int qmla_mla_decode_pair(const void* pool_dev, int c_bits, int num_blocks, const uint16_t* q_latent_dev,
+                         const uint16_t* q_pe_dev, int batch, int q_tokens, int heads,
+                         const int32_t* block_table_dev, int max_blocks, const int32_t* seq_lens_dev,
+                         float softmax_scale, float* out_dev, float* lse_dev, void* workspace_dev,
+                         size_t workspace_bytes, uint32_t* dev_err_dev, qmla_stream_t stream);
+
 /* The same decode over the BF16 comparison cache (same kernel, no dequantisation;
  * the paper's BF16 baseline, App. F.1). */
 int qmla_mla_decode_bf16cache(const void* pool_dev, int num_blocks, const uint16_t* q_latent_dev,

@@ -76,6 +76,9 @@ def lib():
     L.qmla_mla_decode_multi.argtypes = [vp, i32, i32, vp, vp, i32, i32, i32, vp, i32, vp, vp, f32, vp, vp, vp, sz,
                                         vp, vp]
     L.qmla_mla_decode_multi.restype = i32
+    L.qmla_mla_decode_pair.argtypes = [vp, i32, i32, vp, vp, i32, i32, i32, vp, i32, vp, f32, vp, vp, vp, sz, vp,
+                                       vp]
+    L.qmla_mla_decode_pair.restype = i32
     L.qmla_debug_wait_timeout.argtypes = [ctypes.c_uint32, vp, vp]
     L.qmla_debug_wait_timeout.restype = i32
     L.qmla_debug_tile.argtypes = [vp, i32, i32, vp, i32, vp, i32, i32, i32, vp, vp, vp, vp]
@@ -200,6 +203,22 @@ def mla_decode_multi(pool: torch.Tensor, c_bits: int, q_latent: torch.Tensor, q_
                                      float(softmax_scale), _ptr(out), _ptr(lse), _ptr(workspace),
                                      workspace.numel() * workspace.element_size(), _ptr(dev_err), _stream(stream))
     _check("qmla_mla_decode_multi", st)
+
+
+def mla_decode_pair(pool: torch.Tensor, c_bits: int, q_latent: torch.Tensor, q_pe: torch.Tensor,
+                    block_table: torch.Tensor, seq_lens: torch.Tensor, softmax_scale: float, out: torch.Tensor,
+                    lse: torch.Tensor | None, workspace: torch.Tensor, dev_err: torch.Tensor, stream=None) -> None:
+    """qmla_mla_decode_pair: the decode on CTA pairs for q_tokens x heads a multiple of 128.
+    q_latent bf16 [B,H,512] or [B,T,H,512] (out, lse likewise); workspace for B x (T*H) heads."""
+    if q_latent.dim() == 3:
+        B, T, H = q_latent.shape[0], 1, q_latent.shape[1]
+    else:
+        B, T, H = q_latent.shape[0], q_latent.shape[1], q_latent.shape[2]
+    st = lib().qmla_mla_decode_pair(_ptr(pool), c_bits, pool.shape[0], _ptr(q_latent), _ptr(q_pe), B, T, H,
+                                    _ptr(block_table), block_table.shape[1], _ptr(seq_lens), float(softmax_scale),
+                                    _ptr(out), _ptr(lse), _ptr(workspace),
+                                    workspace.numel() * workspace.element_size(), _ptr(dev_err), _stream(stream))
+    _check("qmla_mla_decode_pair", st)
 
 
 CACHE_C4R4 = 5   # qmla_debug_tile cache kinds (besides content bit widths 4 and 2)

@@ -63,7 +63,8 @@ int append_common_checks(const void* pool, int num_blocks, const uint16_t* laten
 int decode_common(const void* pool, int kind, int num_blocks, const uint16_t* q_latent, const uint16_t* q_pe,
                   int batch, int heads, const int32_t* table, int max_blocks, const int32_t* seq_lens,
                   float softmax_scale, float* out, float* lse, void* workspace, size_t workspace_bytes,
-                  uint32_t* dev_err, qmla_stream_t stream, const void* prot = nullptr, int q_tokens = 1) {
+                  uint32_t* dev_err, qmla_stream_t stream, const void* prot = nullptr, int q_tokens = 1,
+                  bool pair = false) {
   if (pool == nullptr || q_latent == nullptr || q_pe == nullptr || table == nullptr || seq_lens == nullptr ||
       out == nullptr || workspace == nullptr)
     return QMLA_ERR_INVALID_ARG;
@@ -103,6 +104,7 @@ int decode_common(const void* pool, int kind, int num_blocks, const uint16_t* q_
   a.q_tokens = q_tokens;
   a.ev_before_main = g_ev_before_main;
   a.ev_after_main = g_ev_after_main;
+  a.pair = pair;
   cudaError_t e = qmla::launch_decode(a, reinterpret_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
 }
@@ -251,6 +253,19 @@ int qmla_mla_decode_multi(const void* pool_dev, int c_bits, int num_blocks, cons
   return decode_common(pool_dev, c_bits, num_blocks, q_latent_dev, q_pe_dev, batch, q_tokens * heads,
                        block_table_dev, max_blocks, seq_lens_dev, softmax_scale, out_dev, lse_dev, workspace_dev,
                        workspace_bytes, dev_err_dev, stream, prot_dev, q_tokens);
+}
+
+int qmla_mla_decode_pair(const void* pool_dev, int c_bits, int num_blocks, const uint16_t* q_latent_dev,
+                         const uint16_t* q_pe_dev, int batch, int q_tokens, int heads,
+                         const int32_t* block_table_dev, int max_blocks, const int32_t* seq_lens_dev,
+                         float softmax_scale, float* out_dev, float* lse_dev, void* workspace_dev,
+                         size_t workspace_bytes, uint32_t* dev_err_dev, qmla_stream_t stream) {
+  if (c_bits != 4 && c_bits != 2) return QMLA_ERR_INVALID_ARG;
+  if (q_tokens < 1 || q_tokens > QMLA_MAX_Q_TOKENS || heads < 1 || heads > 128) return QMLA_ERR_INVALID_ARG;
+  if ((q_tokens * heads) % 128 != 0) return QMLA_ERR_UNSUPPORTED;
+  return decode_common(pool_dev, c_bits, num_blocks, q_latent_dev, q_pe_dev, batch, q_tokens * heads,
+                       block_table_dev, max_blocks, seq_lens_dev, softmax_scale, out_dev, lse_dev, workspace_dev,
+                       workspace_bytes, dev_err_dev, stream, nullptr, q_tokens, true);
 }
 
 int qmla_mla_decode_bf16cache(const void* pool_dev, int num_blocks, const uint16_t* q_latent_dev,

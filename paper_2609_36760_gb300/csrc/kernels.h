@@ -47,6 +47,9 @@ struct DecodeArgs {
   const void* prot = nullptr;  // sink4/local128 protection buffer, or null
   cudaEvent_t ev_before_main = nullptr;  // optional, recorded around the main kernel
   cudaEvent_t ev_after_main = nullptr;
+  // Cluster-pair kernel: units of 128 query rows (heads a multiple of 128),
+  // cache_kind 4 or 2, no protection buffer.
+  bool pair = false;
 };
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
 // Test hook: tile j of sequence b as the decode kernel builds it, [128][576] fp16.
