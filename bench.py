@@ -58,6 +58,9 @@ def parse(argv=None):
     ap.add_argument("--pair", action="store_true",
                     help="decode on CTA pairs (qmla_mla_decode_pair; heads x q-tokens a multiple of 128, "
                          "INT4/INT2 block, no protection)")
+    ap.add_argument("--trace", default=None, metavar="NPZ",
+                    help="instead of timing: build the trace library, trace one decode step's main kernel, print "
+                         "the per-tile stage breakdown and save the raw clock64 stamps to NPZ")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args(argv)
@@ -617,8 +620,82 @@ def run_reference(args, ws_world: int, rank: int):
     print(json.dumps(res), flush=True)
 
 
+TRACE_CTAS, TRACE_EVENTS, TRACE_TILES = 8, 128, 32
+
+
+def run_trace(args):
+    """Per-tile event timeline of the main decode kernel from the trace build
+    (-DQMLA_TRACE_BUILD: clock64 stamps at pipeline events of the first eight
+    CTAs, written through the buffer given to qmla_trace_set). Stamps are per-SM
+    clocks: only differences within one CTA mean anything. Events of the
+    CTA-pair kernel: MMA thread 0 loop top, 4 QK issued, 1 QK committed, 2 P
+    seen, 3 PV committed; lane 0 of warp 0 at 8 + k and of warp 2 at 16 + k,
+    k = 0 loop top, 1 next tile dequantised, 2 previous segment written, 3
+    scores seen, 4 peer scores seen (owner) / scores sent (relay), 5 max agreed
+    (owner) / peer P seen (relay), 6 P sent (owner), 7 P in TMEM; rank 0 owns
+    the heads of warp 0, rank 1 those of warp 2."""
+    import ctypes
+
+    import numpy as np
+
+    from paper_2609_36760_gb300 import build as B
+    lib_path = B.build(trace=True)
+    import paper_2609_36760_gb300 as Q
+    Q._LIB_PATH = lib_path  # the traced library, loaded before any other call
+    L = Q.lib()
+    L.qmla_trace_set.argtypes, L.qmla_trace_set.restype = [ctypes.c_void_p], ctypes.c_int
+    dev = torch.device("cuda", 0)
+    st = Workspace(W.WORKLOADS[args.workload], args.bf16_cache, dev, 4, protect=args.protect, c4r4=args.c4r4,
+                   q_tokens=args.q_tokens, pair=args.pair)
+    buf = torch.zeros(TRACE_CTAS * TRACE_EVENTS * TRACE_TILES + 4 * 1024, dtype=torch.int64, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    for i in range(3):
+        flush.zero_()
+        st.step(i)
+    L.qmla_trace_set(ctypes.c_void_p(buf.data_ptr()))
+    flush.zero_()
+    st.step(3)
+    torch.cuda.synchronize()
+    L.qmla_trace_set(None)
+    if Q.read_dev_err(st.err) != 0:
+        raise SystemExit(f"device error word {Q.read_dev_err(st.err):#x}")
+    t = buf.cpu().numpy()
+    np.savez(args.trace, t=t)
+    ev = t[:TRACE_CTAS * TRACE_EVENTS * TRACE_TILES].reshape(TRACE_CTAS, TRACE_EVENTS, TRACE_TILES)
+    cta = t[TRACE_CTAS * TRACE_EVENTS * TRACE_TILES:].reshape(-1, 4)
+    live = cta[cta[:, 0] > 0]
+    print(f"CTAs {len(live)}, wall us {(live[:, 1] - live[:, 0]).min() / 1e3:.1f} .. "
+          f"{(live[:, 1] - live[:, 0]).max() / 1e3:.1f}, tiles per CTA {live[:, 3].min()} .. {live[:, 3].max()}")
+    if not args.pair:
+        print(f"raw stamps saved to {args.trace} (decode_main's event numbers are in decode.cu)")
+        return
+    stages, period = {}, []
+    for c in range(TRACE_CTAS):
+        n = int((ev[c, 0] > 0).sum())
+        period += list(np.diff(ev[c, 0, :n])[2:])
+        own, rel = (8, 16) if c % 2 == 0 else (16, 8)
+        for it in range(2, n - 1):
+            g = ev[c, :, it]
+            for name, v in (("mma: loop top -> QK issued", g[4] - g[0]), ("mma: QK committed -> P seen", g[2] - g[1]),
+                            ("mma: P seen -> PV committed", g[3] - g[2]),
+                            ("owner: next tile dequantised", g[own + 1] - g[own]),
+                            ("owner: scores seen -> peer scores", g[own + 4] - g[own + 3]),
+                            ("owner: max agreed", g[own + 5] - g[own + 4]),
+                            ("owner: P computed and sent", g[own + 6] - g[own + 5]),
+                            ("owner: P in TMEM", g[own + 7] - g[own + 6]),
+                            ("relay: scores sent", g[rel + 4] - g[rel + 3]),
+                            ("relay: waiting for the peer's P", g[rel + 5] - g[rel + 4])):
+                stages.setdefault(name, []).append(v)
+    print(f"tile period (cycles, median): {np.median(period):.0f}")
+    for k, v in stages.items():
+        print(f"  {k:36s} {np.median(v):7.0f}")
+
+
 def main():
     args = parse()
+    if args.trace:
+        run_trace(args)
+        return
     ws_world, rank, local = dist_env()
     if args.impl == "reference":
         run_reference(args, ws_world, rank)

@@ -289,6 +289,12 @@ __device__ bool epilogue(const Params& p, const SegEnd& e, Ctl& c, uint32_t t_ro
 // column half th = w >> 2. Dequantises token row 32 q + lane of its chunks;
 // in the softmax step it either owns its heads (q >> 1 == rank) or relays
 // them to and from the peer.
+// Trace builds: lane 0 of warps 0 and 2 records events 8.. and 16.. per tile.
+#define PAIR_TRACE(k)                                                            \
+  do {                                                                           \
+    if (lane == 0 && (warp == 0 || warp == 2)) QMLA_TRACE(8 + 4 * warp + (k), it); \
+  } while (0)
+
 template <int CB>
 __device__ void worker_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, uint32_t tmem, uint32_t rank,
                             const Peer& pr, int pair_id, int warp, int lane) {
@@ -355,6 +361,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, u
   for (; ok && sc.valid(); sc.next()) {
     const TileFlags tf = tile_flags(sc);
     if (tf.first) seg_j0 = sc.t - sc.pu0;
+    PAIR_TRACE(0);
     // ---- tile it + 1 into buffer (it + 1) & 1 once the PV of tile it - 1 read it
     if (s1.valid()) {
       const uint32_t nb = (it + 1) & 1u;
@@ -370,6 +377,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, u
     s1 = s2;
     s2.next();
     r2 = row_ref(p, s2, row);
+    PAIR_TRACE(1);
 
     // ---- the previous segment's results once its last PV has completed
     if (pending) {
@@ -380,8 +388,10 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, u
     }
 
     // ---- scores of this tile
+    PAIR_TRACE(2);
     if (!(ok = pwait(&c.s_full, it & 1u, c, pr, kPsS, p.dev_err))) break;
     tc_fence_after();
+    PAIR_TRACE(3);
     const TileInfo ti = tile_info(sc, p);
     uint32_t s[64];
     tmem_ld64(t_row + kColS + 64 * th, s);
@@ -395,6 +405,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, u
       const int tq = v / p.hpt;
       const int lim = min(max(ti.len - p.q_tokens + tq - kTileTokens * ti.j - 64 * th + 1, 0), 64);
       if (!(ok = pwait(&c.srecv_full, it & 1u, c, pr, kPsSrecv, p.dev_err, true))) break;
+      PAIR_TRACE(4);
       float x[64];
       float mx = -INFINITY;
 #pragma unroll
@@ -411,6 +422,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, u
       const uint32_t up = nq & 1u;
       c.red[up][q][th][lane] = mx;
       if (!(ok = quarter_sync(c, q, nq, pr, p.dev_err, lane))) break;
+      PAIR_TRACE(5);
       const float M = fmaxf(c.red[up][q][0][lane], c.red[up][q][1][lane]);
       if (ti.first) {
         m_ref = M;  // new segment: the reference is this tile's max
@@ -427,13 +439,16 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, u
       for (int tg = 0; tg < 8; ++tg) st_cluster_v4(pr_peer + tg * 512, pk[4 * tg], pk[4 * tg + 1], pk[4 * tg + 2], pk[4 * tg + 3]);
       st_cluster_u32(al_peer, __float_as_uint(alpha));
       mbar_arrive_cluster(prb_peer);
+      PAIR_TRACE(6);
     } else {
       // Relay: this CTA's partial scores of the peer's heads to the peer, then
       // the peer's P of those heads into this CTA's TMEM.
 #pragma unroll
       for (int tg = 0; tg < 16; ++tg) st_cluster_v4(sr_peer + tg * 512, s[4 * tg], s[4 * tg + 1], s[4 * tg + 2], s[4 * tg + 3]);
       mbar_arrive_cluster(srb_peer);
+      PAIR_TRACE(4);
       if (!(ok = pwait(&c.precv_full, it & 1u, c, pr, kPsPrecv, p.dev_err, true))) break;
+      PAIR_TRACE(5);
       alpha = lds_f32(al_loc);
 #pragma unroll
       for (int tg = 0; tg < 8; ++tg) {
@@ -453,6 +468,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, u
     tc_fence_before();
     __syncwarp();
     mbar_arrive_if(lane == 0 ? 1u : 0u, &c.p_full);
+    PAIR_TRACE(7);
 
     if (ti.last) {
       pending = true;
@@ -500,6 +516,7 @@ __device__ void mma_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, uint
     const TileFlags tf = tile_flags(sc);
     const uint32_t b = it & 1u;
     const uint64_t boff = static_cast<uint64_t>((b * kBufBytes) >> 4);
+    QMLA_TRACE(0, it);
     if (tf.first && !(ok = twait(&c.q_full, seg & 1u, c, pr, kPsQ, p.dev_err))) break;
     if (!(ok = twait(&c.full[b], (it >> 1) & 1u, c, pr, kPsFull, p.dev_err))) break;
     // S and P share TMEM columns: the previous tile's PV must have read its P.
@@ -514,8 +531,11 @@ __device__ void mma_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, uint
     for (int ks = 0; ks < 2; ++ks)
       umma_f16_ss(t_s, pe_a0 + static_cast<uint64_t>((ks * 32) >> 4),
                   pe_b0 + boff + static_cast<uint64_t>((ks * 32) >> 4), kIdQK, 1u);
+    QMLA_TRACE(4, it);
     umma_commit(&c.s_full);
+    QMLA_TRACE(1, it);
     if (!(ok = twait(&c.p_full, it & 1u, c, pr, kPsP, p.dev_err))) break;
+    QMLA_TRACE(2, it);
     if (tf.first && seg > 0 && !(ok = twait(&c.o_free, (seg - 1) & 1u, c, pr, kPsO, p.dev_err))) break;
     tc_fence_after();
     const uint32_t acc0 = tf.first ? 0u : 1u;
@@ -524,6 +544,7 @@ __device__ void mma_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, uint
       umma_f16_ts(t_o, t_s + 64 * (ks >> 2) + 8 * (ks & 3), pv_b0 + boff + static_cast<uint64_t>((ks * 2048) >> 4),
                   kIdPV, ks > 0 ? 1u : acc0);
     umma_commit(&c.empty[b]);
+    QMLA_TRACE(3, it);
     ++it;
     if (tf.last) ++seg;
   }
@@ -544,6 +565,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_pair(const Params p) {
   const int lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
   const int pair_id = static_cast<int>(blockIdx.x >> 1);
+  if (threadIdx.x == 0) {
+    QMLA_TRACE_CTA(0, globaltimer_ns());
+    uint32_t smid;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(smid));
+    QMLA_TRACE_CTA(2, smid);
+  }
   if (threadIdx.x == 0) {
     for (int b = 0; b < 2; ++b) {
       mbar_init(&c.full[b], kWorkers);
@@ -598,8 +625,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_pair(const Params p) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
+  if (threadIdx.x == 0) {
+    QMLA_TRACE_CTA(1, globaltimer_ns());
+    QMLA_TRACE_CTA(3, static_cast<unsigned long long>(sc.t1 - sc.t0));
+  }
 }
 
+#undef PAIR_TRACE
 }  // namespace pairk
 
 // Launches kern with clusters of two CTAs (and programmatic stream
