@@ -629,17 +629,20 @@ def run_trace(args):
     CTAs, written through the buffer given to qmla_trace_set). Stamps are per-SM
     clocks: only differences within one CTA mean anything. Events of the
     CTA-pair kernel: MMA thread 0 loop top, 4 QK issued, 1 QK committed, 2 P
-    seen, 3 PV committed; lane 0 of warp 0 at 8 + k and of warp 2 at 16 + k,
-    k = 0 loop top, 1 next tile dequantised, 2 previous segment written, 3
-    scores seen, 4 peer scores seen (owner) / scores sent (relay), 5 max agreed
-    (owner) / peer P seen (relay), 6 P sent (owner), 7 P in TMEM; rank 0 owns
-    the heads of warp 0, rank 1 those of warp 2."""
+    seen, 3 PV committed; lane 0 of softmax warps 0 and 2 at 8 + k and 16 + k,
+    k = 0 loop top, 3 scores seen, 4 relayed scores sent and own scores read,
+    5 peer scores added and the tile max agreed in the CTA, 6 P and max sent,
+    7 P in TMEM (after the peer's P, and a second exchange when the reference
+    moved)."""
     import ctypes
 
     import numpy as np
 
     from paper_2609_36760_gb300 import build as B
-    lib_path = B.build(trace=True)
+    lib_path = os.path.join(B.LIBDIR, "libqmla_trace.so")
+    srcs = [os.path.join(B.CSRC, f) for f in os.listdir(B.CSRC)] + [os.path.join(B.INCLUDE, "qmla.h")]
+    if not os.path.exists(lib_path) or max(map(os.path.getmtime, srcs)) > os.path.getmtime(lib_path):
+        lib_path = B.build(trace=True)
     import paper_2609_36760_gb300 as Q
     Q._LIB_PATH = lib_path  # the traced library, loaded before any other call
     L = Q.lib()
@@ -673,19 +676,18 @@ def run_trace(args):
     for c in range(TRACE_CTAS):
         n = int((ev[c, 0] > 0).sum())
         period += list(np.diff(ev[c, 0, :n])[2:])
-        own, rel = (8, 16) if c % 2 == 0 else (16, 8)
         for it in range(2, n - 1):
             g = ev[c, :, it]
             for name, v in (("mma: loop top -> QK issued", g[4] - g[0]), ("mma: QK committed -> P seen", g[2] - g[1]),
-                            ("mma: P seen -> PV committed", g[3] - g[2]),
-                            ("owner: next tile dequantised", g[own + 1] - g[own]),
-                            ("owner: scores seen -> peer scores", g[own + 4] - g[own + 3]),
-                            ("owner: max agreed", g[own + 5] - g[own + 4]),
-                            ("owner: P computed and sent", g[own + 6] - g[own + 5]),
-                            ("owner: P in TMEM", g[own + 7] - g[own + 6]),
-                            ("relay: scores sent", g[rel + 4] - g[rel + 3]),
-                            ("relay: waiting for the peer's P", g[rel + 5] - g[rel + 4])):
+                            ("mma: P seen -> PV committed", g[3] - g[2])):
                 stages.setdefault(name, []).append(v)
+            for w0 in (8, 16):
+                for name, v in (("softmax: loop top -> scores seen", g[w0 + 3] - g[w0]),
+                                ("softmax: relay sent, own read", g[w0 + 4] - g[w0 + 3]),
+                                ("softmax: peer scores, max agreed", g[w0 + 5] - g[w0 + 4]),
+                                ("softmax: P and max sent", g[w0 + 6] - g[w0 + 5]),
+                                ("softmax: peer P, P in TMEM", g[w0 + 7] - g[w0 + 6])):
+                    stages.setdefault(name, []).append(v)
     print(f"tile period (cycles, median): {np.median(period):.0f}")
     for k, v in stages.items():
         print(f"  {k:36s} {np.median(v):7.0f}")

@@ -18,17 +18,22 @@
 //        16 MMAs with A = q from TMEM, B = the content chunks (K-major), and two
 //        with A = the RoPE query half, B = the RoPE half chunk (both in shared
 //        memory, 64-byte swizzle); M = 128 heads, N = 128 tokens.
-//   Each CTA owns 64 heads (lanes 64 r .. 64 r + 63). The warps on the other
-//   lanes send those heads' partial scores to the peer (distributed shared
-//   memory); the warps on the owned lanes add the peer's partial for their
-//   heads, keep the per-head reference max (raised only when a score exceeds
-//   it by 2^8, as in decode_main), form P = 2^(S scale log2e - m) in fp16, store
-//   it into TMEM and send it, with the rescale factor, to the peer, whose warps
-//   on those lanes store it into its TMEM.
+//   Softmax, split by tokens: CTA r owns tokens [64 r, 64 r + 64) of the tile
+//   for all 128 heads. Softmax warp (q, hh) (TMEM lane quarter q: heads
+//   32 q .. 32 q + 31) owns the 32 tokens 64 r + 32 hh .. and sends this CTA's
+//   partial scores of the peer's 32 tokens 64 (1 - r) + 32 hh .. to the peer's
+//   warp (q, hh) (distributed shared memory), adds the peer's partial for its
+//   own tokens, agrees the tile max with its partner warp and, through the P
+//   message, with the peer, forms P = 2^(S scale log2e - m) in fp16 against the
+//   per-head reference m (raised only when a score exceeds it by 2^8, as in
+//   decode_main; P is sent optimistically against the current reference and
+//   re-sent in the rare tile that raises it) and writes its own and the peer's
+//   P over the scores in TMEM. Both CTAs sum the same fp16 weights in the same
+//   order, so both hold the same row sums.
 //   PV   O_r[h, c] += sum_t P[h, t] C_hat[t, c]: 8 MMAs with A = P from TMEM,
 //        B = the same content chunks read MN-major, N = 256 channels.
-// The reconstructed tile is double-buffered: the next tile is dequantised while
-// this one is in QK and softmax. Every wait is bounded; a wait that runs out
+// Dedicated warps dequantise the next tile into the second buffer while this
+// one is in QK and softmax. Every wait is bounded; a wait that runs out
 // records its site, stops both CTAs of the pair and they leave.
 namespace pairk {
 
@@ -37,27 +42,32 @@ constexpr int kCChunks = 4;                                     // content chunk
 constexpr int kRopeRow = 64;                                    // bytes per row of the RoPE half
 constexpr int kBufBytes = kCChunks * kChunkBytes + kTileTokens * kRopeRow;  // 73728
 constexpr int kQRopeBytes = kHeads * kRopeRow;                  // 8192
-constexpr int kSrecvBytes = 64 * kTileTokens * 4;               // peer partial scores of the owned heads
-constexpr int kPrecvBytes = 64 * kTileTokens * 2;               // peer P of the other heads
-constexpr int kAlphaBytes = 4 * 32 * 4;                         // peer rescale factors
+constexpr int kSWarps = 8;                                      // softmax warps (lane quarter x token half)
+constexpr int kDqWarps = 4;                                     // dequantisation warps (a token row per thread)
+constexpr int kPairMmaWarp = kSWarps + kDqWarps;                // one thread issues the MMAs
+constexpr int kPairThreads = (kPairMmaWarp + 1) * 32;           // 416
+constexpr int kSrecvBytes = kSWarps * 32 * 32 * 4;              // peer partial scores: [warp][8][lane][4 fp32]
+constexpr int kPrecvBytes = kSWarps * 32 * 16 * 4;              // peer P: [warp][4][lane][8 fp16]
+constexpr int kMrecvBytes = kSWarps * 32 * 4;                   // peer tile max: [warp][lane]
 constexpr uint32_t kColO = 0, kColS = 256, kColQ = 384, kTmemCols = 512;
 constexpr int kOffQRope = 2 * kBufBytes;
 constexpr int kOffSrecv = kOffQRope + kQRopeBytes;
 constexpr int kOffPrecv = kOffSrecv + kSrecvBytes;
-constexpr int kOffAlpha = kOffPrecv + kPrecvBytes;
-constexpr int kOffCtrl = kOffAlpha + kAlphaBytes;
+constexpr int kOffMrecv = kOffPrecv + kPrecvBytes;
+constexpr int kOffCtrl = kOffMrecv + kMrecvBytes;
 static_assert(kBufBytes % 1024 == 0 && kOffQRope % 1024 == 0, "swizzle atom alignment");
 static_assert((kCChunks * kChunkBytes) % 512 == 0, "64-byte swizzle alignment of the RoPE half");
 
 struct __align__(16) Ctl {
-  // full[b]: the tile in buffer b is dequantised (one arrive per worker warp).
+  // full[b]: the tile in buffer b is dequantised (one arrive per dequantisation warp).
   // empty[b]: the PV that read buffer b has completed (MMA commit).
   uint64_t full[2], empty[2];
   uint64_t s_full, p_full, q_full, o_free, fin;
-  // Arrived on by the peer: its partial scores / its P and factors are here
-  // (one arrive per sending thread); done: the peer no longer touches this CTA.
-  uint64_t srecv_full, precv_full, done;
-  uint64_t qbar[4];  // the two warps of a TMEM lane quarter
+  // Arrived on by the peer's softmax warp w (every lane): its partial scores,
+  // its P and tile max, its P again after a raised reference; done: the peer
+  // no longer touches this CTA.
+  uint64_t srecv[kSWarps], precv[kSWarps], precv2[kSWarps], done;
+  uint64_t qbar[4];  // the two softmax warps of a TMEM lane quarter
   uint32_t tmem_base;
   uint32_t abort;
   alignas(16) float red[2][4][2][32];  // [use parity][lane quarter][token half][lane]
@@ -225,22 +235,29 @@ __device__ __forceinline__ void scale_o(uint32_t t_o, float a) {
   tmem_st_wait();
 }
 
-// Adds the 64 fp16 weights of pk to l in a fixed order (the owner and the
-// peer's relaying thread sum the same values the same way, so both hold the
-// same row sum).
-__device__ __forceinline__ float add_weights(float l, const uint32_t (&pk)[32]) {
+// Adds 16 words of fp16 weight pairs to l in a fixed order (both CTAs sum
+// the same values the same way, so both hold the same row sum).
+__device__ __forceinline__ float add_weights(float l, const uint32_t (&w)[16]) {
 #pragma unroll
-  for (int k = 0; k < 32; ++k) {
-    const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&pk[k]));
+  for (int k = 0; k < 16; ++k) {
+    const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w[k]));
     l += f.x;
     l += f.y;
   }
   return l;
 }
 
+// P of 32 scaled scores against the reference m: 2^(x - m) in fp16 pairs,
+// 0 for the tokens at or past lim (masked or past the sequence end).
+__device__ __forceinline__ void weights(uint32_t (&pk)[16], const float (&x)[32], float m, int lim) {
+#pragma unroll
+  for (int k = 0; k < 16; ++k)
+    pk[k] = pack_h2(2 * k < lim ? ex2_approx(x[2 * k] - m) : 0.0f, 2 * k + 1 < lim ? ex2_approx(x[2 * k + 1] - m) : 0.0f);
+}
+
 // Segment end for the thread of head h (lane quarter q) and column half th:
 // l = both token halves' row sums, then out = O / l over the CTA's channels
-// (or the unnormalised partial), and LSE / (m, l) from the owner.
+// (or the unnormalised partial), and LSE / (m, l) from `owner` (rank 0).
 template <int CB>
 __device__ bool epilogue(const Params& p, const SegEnd& e, Ctl& c, uint32_t t_row, uint32_t rank, bool owner,
                          int q, int th, int lane, float m_ref, float l_half, uint32_t& nq, const Peer& pr) {
@@ -284,48 +301,43 @@ __device__ bool epilogue(const Params& p, const SegEnd& e, Ctl& c, uint32_t t_ro
   return true;
 }
 
-// ------------------------------------------------------------ worker warps
-// Warp w: TMEM lane quarter q = w & 3 (heads 32 q .. 32 q + 31), token half /
-// column half th = w >> 2. Dequantises token row 32 q + lane of its chunks;
-// in the softmax step it either owns its heads (q >> 1 == rank) or relays
-// them to and from the peer.
-// Trace builds: lane 0 of warps 0 and 2 records events 8.. and 16.. per tile.
-#define PAIR_TRACE(k)                                                            \
-  do {                                                                           \
-    if (lane == 0 && (warp == 0 || warp == 2)) QMLA_TRACE(8 + 4 * warp + (k), it); \
-  } while (0)
-
+// ------------------------------------------------------- dequantisation
+// Packed rows of one token for every chunk of this CTA's half: content chunks
+// 0..3 and the RoPE-key half.
+struct RowsAll {
+  Fetch c[kCChunks];
+  Fetch pe;
+};
 template <int CB>
-__device__ void worker_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, uint32_t tmem, uint32_t rank,
-                            const Peer& pr, int pair_id, int warp, int lane) {
-  const int q = warp & 3, th = warp >> 2;
-  const int h = 32 * q + lane;
-  const int row = h, slot = row & 63;
-  const bool owner = (q >> 1) == static_cast<int>(rank);
-  const int blk = (q & 1) * 2 + th;  // block of the exchange buffers
-  const uint32_t t_row = tmem + (static_cast<uint32_t>(32 * q) << 16);
-  const uint32_t sr_loc = sbase + kOffSrecv + blk * 8192 + lane * 16;  // + 512 per 4 tokens
-  const uint32_t pr_loc = sbase + kOffPrecv + blk * 4096 + lane * 16;  // + 512 per 8 tokens
-  const uint32_t al_loc = sbase + kOffAlpha + (blk * 32 + lane) * 4;
-  const uint32_t sr_peer = cluster_map(sr_loc, pr.rank);
-  const uint32_t pr_peer = cluster_map(pr_loc, pr.rank);
-  const uint32_t al_peer = cluster_map(al_loc, pr.rank);
-  const uint32_t srb_peer = cluster_map(smem_u32(&c.srecv_full), pr.rank);
-  const uint32_t prb_peer = cluster_map(smem_u32(&c.precv_full), pr.rank);
-  const uint32_t qrope = sbase + kOffQRope;
-  const float sl2 = p.scale_log2;
-  uint32_t it = 0, nq = 0;
-  float m_ref = -INFINITY, l_half = 0.0f;
-  int seg_j0 = 0;
-  bool ok = true, pending = false;
-  SegEnd pend{};
-  if (!sc.valid()) return;
+__device__ __forceinline__ void fetch_all(RowsAll& f, const uint8_t* blk, bool valid, uint32_t rank, int slot) {
+  Rows h;
+#pragma unroll
+  for (int th = 0; th < 2; ++th) {
+    fetch_rows<CB>(h, blk, valid, rank, th, slot);
+    f.c[th] = h.c0;
+    f.c[th + 2] = h.c1;
+    if (th == 0) f.pe = h.pe;
+  }
+}
+template <int CB>
+__device__ __forceinline__ void store_all(const RowsAll& f, uint32_t buf, int row) {
+#pragma unroll
+  for (int i = 0; i < kCChunks; ++i) store_row<CB>(buf + i * kChunkBytes, row, f.c[i], CB == 4);
+  store_rope_half(buf + kCChunks * kChunkBytes, row, f.pe);
+}
 
-  // Tile 0 into buffer 0 (the prep kernel found its table entries), tile 1's
-  // rows into registers, tile 2's table entries, the first unit's queries.
-  Rows f;
+// Dequantisation warp d: token row 32 d + lane of every chunk. Tile `it` goes
+// into buffer it & 1 once the PV of tile it - 2 has read that buffer; the
+// packed rows of the next tile are loaded a tile ahead, its block-table
+// entries a tile before that.
+template <int CB>
+__device__ void dequant_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, uint32_t rank, const Peer& pr,
+                             int pair_id, int d, int lane) {
+  const int row = 32 * d + lane, slot = row & 63;
+  if (!sc.valid()) return;
+  RowsAll f;
   {
-    const int4 fr = p.cta_first[pair_id];
+    const int4 fr = p.cta_first[pair_id];  // tile 0's table entries, from the prep kernel
     RowRef r0;
     r0.has = true;
     r0.entry = row < 64 ? fr.x : fr.y;
@@ -334,24 +346,66 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, u
     r0.b = sc.u / p.n_hg;
     bool v0 = false;
     const uint8_t* b0 = resolve_row<CB>(p, r0, row, v0);
-    fetch_rows<CB>(f, b0, v0, rank, th, slot);
-    store_rows<CB>(f, sbase, row, th);
-    fence_proxy_async_smem();
-    __syncwarp();
-    mbar_arrive_if(lane == 0 ? 1u : 0u, &c.full[0]);
+    fetch_all<CB>(f, b0, v0, rank, slot);
   }
-  Sched s1 = sc;  // tile it + 1
+  Sched s1 = sc;  // the tile after the one being stored
   s1.next();
-  {
-    const RowRef r1 = row_ref(p, s1, row);
+  RowRef r1 = row_ref(p, s1, row);
+  uint32_t it = 0;
+  for (; sc.valid(); sc.next()) {
+    const uint32_t b = it & 1u;
+    if (!pwait(&c.empty[b], ((it >> 1) & 1u) ^ 1u, c, pr, kPsEmpty, p.dev_err)) break;
+    store_all<CB>(f, sbase + b * kBufBytes, row);
     bool v1 = false;
     const uint8_t* b1 = resolve_row<CB>(p, r1, row, v1);
-    fetch_rows<CB>(f, b1, v1, rank, th, slot);
+    fetch_all<CB>(f, b1, v1, rank, slot);
+    s1.next();
+    r1 = row_ref(p, s1, row);
+    fence_proxy_async_smem();
+    __syncwarp();
+    mbar_arrive_if(lane == 0 ? 1u : 0u, &c.full[b]);
+    ++it;
   }
-  Sched s2 = s1;  // tile it + 2
-  s2.next();
-  RowRef r2 = row_ref(p, s2, row);
-  load_query<CB>(p, sc.u, t_row + kColQ, qrope, rank, h, th);
+}
+
+// ------------------------------------------------------------ softmax warps
+// Trace builds: lane 0 of warps 0 and 2 records events 8.. and 16.. per tile.
+#define PAIR_TRACE(k)                                                            \
+  do {                                                                           \
+    if (lane == 0 && (warp == 0 || warp == 2)) QMLA_TRACE(8 + 4 * warp + (k), it); \
+  } while (0)
+
+// Softmax warp w: TMEM lane quarter q = w & 3 (heads 32 q .. 32 q + 31), token
+// half hh = w >> 2 of each CTA's 64 tokens. Token group g (tokens 32 g ..
+// 32 g + 31 of the tile, K-steps 2 g and 2 g + 1 of the PV) is owned by warp
+// (q, g & 1) of CTA g >> 1; this warp owns group 2 r + hh and relays group
+// 2 (1 - r) + hh. It alone reads the scores of those two groups and writes
+// their P (K-step k at columns 16 k .. 16 k + 7 of the score block), so P
+// never overwrites scores another warp still has to read.
+template <int CB>
+__device__ void softmax_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, uint32_t tmem, uint32_t rank,
+                             const Peer& pr, int pair_id, int warp, int lane) {
+  const int q = warp & 3, hh = warp >> 2;
+  const int h = 32 * q + lane;
+  const int g_own = 2 * static_cast<int>(rank) + hh, g_rel = 2 * (1 - static_cast<int>(rank)) + hh;
+  const uint32_t t_row = tmem + (static_cast<uint32_t>(32 * q) << 16);
+  const uint32_t sr_loc = sbase + kOffSrecv + warp * 4096 + lane * 16;  // + 512 per 4 tokens
+  const uint32_t pr_loc = sbase + kOffPrecv + warp * 2048 + lane * 16;  // + 512 per 8 tokens
+  const uint32_t m_loc = sbase + kOffMrecv + (warp * 32 + lane) * 4;
+  const uint32_t sr_peer = cluster_map(sr_loc, pr.rank);
+  const uint32_t pr_peer = cluster_map(pr_loc, pr.rank);
+  const uint32_t m_peer = cluster_map(m_loc, pr.rank);
+  const uint32_t srb_peer = cluster_map(smem_u32(&c.srecv[warp]), pr.rank);
+  const uint32_t prb_peer = cluster_map(smem_u32(&c.precv[warp]), pr.rank);
+  const uint32_t pr2b_peer = cluster_map(smem_u32(&c.precv2[warp]), pr.rank);
+  const uint32_t qrope = sbase + kOffQRope;
+  const float sl2 = p.scale_log2;
+  uint32_t it = 0, nq = 0, n2 = 0;
+  float m_ref = -INFINITY, l_half = 0.0f;
+  int seg_j0 = 0;
+  bool ok = true;
+  if (!sc.valid()) return;
+  load_query<CB>(p, sc.u, t_row + kColQ, qrope, rank, h, hh);
   tmem_st_wait();
   fence_proxy_async_smem();
   tc_fence_before();
@@ -362,108 +416,100 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, u
     const TileFlags tf = tile_flags(sc);
     if (tf.first) seg_j0 = sc.t - sc.pu0;
     PAIR_TRACE(0);
-    // ---- tile it + 1 into buffer (it + 1) & 1 once the PV of tile it - 1 read it
-    if (s1.valid()) {
-      const uint32_t nb = (it + 1) & 1u;
-      if (!(ok = pwait(&c.empty[nb], (((it + 1) >> 1) & 1u) ^ 1u, c, pr, kPsEmpty, p.dev_err))) break;
-      store_rows<CB>(f, sbase + nb * kBufBytes, row, th);
-      bool v2 = false;
-      const uint8_t* b2 = resolve_row<CB>(p, r2, row, v2);
-      fetch_rows<CB>(f, b2, v2, rank, th, slot);  // tile it + 2
-      fence_proxy_async_smem();
-      __syncwarp();
-      mbar_arrive_if(lane == 0 ? 1u : 0u, &c.full[nb]);
-    }
-    s1 = s2;
-    s2.next();
-    r2 = row_ref(p, s2, row);
-    PAIR_TRACE(1);
-
-    // ---- the previous segment's results once its last PV has completed
-    if (pending) {
-      if (!(ok = pwait(&c.empty[(it - 1) & 1u], ((it - 1) >> 1) & 1u, c, pr, kPsEmpty, p.dev_err))) break;
-      tc_fence_after();
-      if (!(ok = epilogue<CB>(p, pend, c, t_row, rank, owner, q, th, lane, m_ref, l_half, nq, pr))) break;
-      pending = false;
-    }
-
-    // ---- scores of this tile
-    PAIR_TRACE(2);
     if (!(ok = pwait(&c.s_full, it & 1u, c, pr, kPsS, p.dev_err))) break;
     tc_fence_after();
     PAIR_TRACE(3);
     const TileInfo ti = tile_info(sc, p);
-    uint32_t s[64];
-    tmem_ld64(t_row + kColS + 64 * th, s);
+    uint32_t s[32];
+    // this CTA's partial scores of the relayed group to the peer's warp (q, hh)
+    tmem_ld32(t_row + kColS + 32 * g_rel, s);
     tmem_ld_wait();
-    uint32_t pk[32];
-    float alpha = 1.0f;
-    if (owner) {
-      // Visible tokens of this half: positions up to the head's query token
-      // (Eq. mla_compact's causal mask; every cached position for one token).
-      const int v = ti.hg * kHeads + h;
-      const int tq = v / p.hpt;
-      const int lim = min(max(ti.len - p.q_tokens + tq - kTileTokens * ti.j - 64 * th + 1, 0), 64);
-      if (!(ok = pwait(&c.srecv_full, it & 1u, c, pr, kPsSrecv, p.dev_err, true))) break;
-      PAIR_TRACE(4);
-      float x[64];
-      float mx = -INFINITY;
 #pragma unroll
-      for (int tg = 0; tg < 16; ++tg) {
-        const uint4 o = lds_v4(sr_loc + tg * 512);
-        const uint32_t ov[4] = {o.x, o.y, o.z, o.w};
+    for (int tg = 0; tg < 8; ++tg) st_cluster_v4(sr_peer + tg * 512, s[4 * tg], s[4 * tg + 1], s[4 * tg + 2], s[4 * tg + 3]);
+    mbar_arrive_cluster(srb_peer);
+    tmem_ld32(t_row + kColS + 32 * g_own, s);
+    // Visible tokens of the own group: positions up to the head's query token
+    // (Eq. mla_compact's causal mask; every cached position for one token).
+    const int tq = (ti.hg * kHeads + h) / p.hpt;
+    const int lim = min(max(ti.len - p.q_tokens + tq - kTileTokens * ti.j - 32 * g_own + 1, 0), 32);
+    tmem_ld_wait();
+    PAIR_TRACE(4);
+    if (!(ok = pwait(&c.srecv[warp], it & 1u, c, pr, kPsSrecv, p.dev_err, true))) break;
+    float x[32];
+    float mx = -INFINITY;
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int i = 4 * tg + e;
-          x[i] = (__uint_as_float(s[i]) + __uint_as_float(ov[e])) * sl2;
-          if (i < lim) mx = fmaxf(mx, x[i]);
-        }
-      }
-      const uint32_t up = nq & 1u;
-      c.red[up][q][th][lane] = mx;
-      if (!(ok = quarter_sync(c, q, nq, pr, p.dev_err, lane))) break;
-      PAIR_TRACE(5);
-      const float M = fmaxf(c.red[up][q][0][lane], c.red[up][q][1][lane]);
-      if (ti.first) {
-        m_ref = M;  // new segment: the reference is this tile's max
-      } else if (M > m_ref + kRescaleLog2) {
-        alpha = exp2f(m_ref - M);  // 0 when no key was seen yet (m_ref = -inf)
-        m_ref = M;
-      }
+    for (int tg = 0; tg < 8; ++tg) {
+      const uint4 o = lds_v4(sr_loc + tg * 512);
+      const uint32_t ov[4] = {o.x, o.y, o.z, o.w};
 #pragma unroll
-      for (int k = 0; k < 32; ++k)
-        pk[k] = pack_h2(2 * k < lim ? ex2_approx(x[2 * k] - m_ref) : 0.0f,
-                        2 * k + 1 < lim ? ex2_approx(x[2 * k + 1] - m_ref) : 0.0f);
-      // P and the factor to the peer's relaying thread of this head.
-#pragma unroll
-      for (int tg = 0; tg < 8; ++tg) st_cluster_v4(pr_peer + tg * 512, pk[4 * tg], pk[4 * tg + 1], pk[4 * tg + 2], pk[4 * tg + 3]);
-      st_cluster_u32(al_peer, __float_as_uint(alpha));
-      mbar_arrive_cluster(prb_peer);
-      PAIR_TRACE(6);
-    } else {
-      // Relay: this CTA's partial scores of the peer's heads to the peer, then
-      // the peer's P of those heads into this CTA's TMEM.
-#pragma unroll
-      for (int tg = 0; tg < 16; ++tg) st_cluster_v4(sr_peer + tg * 512, s[4 * tg], s[4 * tg + 1], s[4 * tg + 2], s[4 * tg + 3]);
-      mbar_arrive_cluster(srb_peer);
-      PAIR_TRACE(4);
-      if (!(ok = pwait(&c.precv_full, it & 1u, c, pr, kPsPrecv, p.dev_err, true))) break;
-      PAIR_TRACE(5);
-      alpha = lds_f32(al_loc);
-#pragma unroll
-      for (int tg = 0; tg < 8; ++tg) {
-        const uint4 o = lds_v4(pr_loc + tg * 512);
-        pk[4 * tg] = o.x;
-        pk[4 * tg + 1] = o.y;
-        pk[4 * tg + 2] = o.z;
-        pk[4 * tg + 3] = o.w;
+      for (int e = 0; e < 4; ++e) {
+        const int i = 4 * tg + e;
+        x[i] = (__uint_as_float(s[i]) + __uint_as_float(ov[e])) * sl2;
+        if (i < lim) mx = fmaxf(mx, x[i]);
       }
     }
-    // (tcgen05.ld / st are warp-collective: the warp rescales when any of its
-    // heads needs it; the others multiply by 1)
-    if (!ti.first && __any_sync(0xffffffffu, alpha != 1.0f)) scale_o(t_row + kColO + 128 * th, alpha);
-    l_half = add_weights(ti.first ? 0.0f : l_half * alpha, pk);
-    tmem_st32(t_row + kColS + 64 * th, pk);
+    // tile max of this CTA's 64 tokens (the partner warp holds the other 32)
+    const uint32_t up = nq & 1u;
+    c.red[up][q][hh][lane] = mx;
+    if (!(ok = quarter_sync(c, q, nq, pr, p.dev_err, lane))) break;
+    const float m_loc_max = fmaxf(c.red[up][q][0][lane], c.red[up][q][1][lane]);
+    PAIR_TRACE(5);
+    // P against the current reference (discarded if the tile raises it), with
+    // the local tile max, to the peer's warp (q, hh)
+    uint32_t pk[16];
+    if (ti.first) {
+#pragma unroll
+      for (int k = 0; k < 16; ++k) pk[k] = 0u;
+    } else {
+      weights(pk, x, m_ref, lim);
+    }
+#pragma unroll
+    for (int tg = 0; tg < 4; ++tg) st_cluster_v4(pr_peer + tg * 512, pk[4 * tg], pk[4 * tg + 1], pk[4 * tg + 2], pk[4 * tg + 3]);
+    st_cluster_u32(m_peer, __float_as_uint(m_loc_max));
+    mbar_arrive_cluster(prb_peer);
+    PAIR_TRACE(6);
+    if (!(ok = pwait(&c.precv[warp], it & 1u, c, pr, kPsPrecv, p.dev_err, true))) break;
+    // The tile max over both CTAs; both compute the same reference.
+    const float M = fmaxf(m_loc_max, lds_f32(m_loc));
+    const bool resc = ti.first || M > m_ref + kRescaleLog2;
+    float alpha = 1.0f;
+    if (__any_sync(0xffffffffu, resc)) {
+      // A new segment, or a score above the reference by more than 2^8 for
+      // some head of this warp: its lanes move the reference (alpha =
+      // 2^(m_old - m_new); 0 when no key was seen yet), recompute P and send
+      // it again; the peer's warp takes the same branch for the same heads.
+      if (resc) {
+        if (!ti.first) alpha = exp2f(m_ref - M);
+        m_ref = M;
+      }
+      weights(pk, x, m_ref, lim);
+#pragma unroll
+      for (int tg = 0; tg < 4; ++tg) st_cluster_v4(pr_peer + tg * 512, pk[4 * tg], pk[4 * tg + 1], pk[4 * tg + 2], pk[4 * tg + 3]);
+      mbar_arrive_cluster(pr2b_peer);
+      // O_r holds the sum through the previous tile (its PV completed before
+      // this tile's QK started) and is scaled to the new reference.
+      if (!ti.first && __any_sync(0xffffffffu, alpha != 1.0f)) scale_o(t_row + kColO + 128 * hh, alpha);
+      if (!(ok = pwait(&c.precv2[warp], n2 & 1u, c, pr, kPsPrecv, p.dev_err, true))) break;
+      ++n2;
+    }
+    uint32_t pp[16];  // the peer's P of the relayed group
+#pragma unroll
+    for (int tg = 0; tg < 4; ++tg) {
+      const uint4 o = lds_v4(pr_loc + tg * 512);
+      pp[4 * tg] = o.x;
+      pp[4 * tg + 1] = o.y;
+      pp[4 * tg + 2] = o.z;
+      pp[4 * tg + 3] = o.w;
+    }
+    // Row sums in group order (group hh, then 2 + hh): the peer's warp (q, hh)
+    // adds the same words in the same order.
+    l_half = ti.first ? 0.0f : l_half * alpha;
+    l_half = add_weights(l_half, rank == 0 ? pk : pp);
+    l_half = add_weights(l_half, rank == 0 ? pp : pk);
+    tmem_st8(t_row + kColS + 32 * g_own, *reinterpret_cast<const uint32_t(*)[8]>(&pk[0]));
+    tmem_st8(t_row + kColS + 32 * g_own + 16, *reinterpret_cast<const uint32_t(*)[8]>(&pk[8]));
+    tmem_st8(t_row + kColS + 32 * g_rel, *reinterpret_cast<const uint32_t(*)[8]>(&pp[0]));
+    tmem_st8(t_row + kColS + 32 * g_rel + 16, *reinterpret_cast<const uint32_t(*)[8]>(&pp[8]));
     tmem_st_wait();
     tc_fence_before();
     __syncwarp();
@@ -471,31 +517,28 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, u
     PAIR_TRACE(7);
 
     if (ti.last) {
-      pending = true;
-      pend.b = ti.b;
-      pend.hg = ti.hg;
-      pend.whole = (seg_j0 == 0) && (sc.t + 1 == sc.pu1);
-      pend.pidx = static_cast<size_t>(pair_id) + sc.u;
-      // The next unit's queries: this tile's QK, the last reader of the
-      // query slice, has completed (s_full above).
+      // The next unit's queries first (this tile's QK, the last reader of the
+      // query slice, has completed), so that its QK can overlap the results.
       Sched nx = sc;
       nx.next();
       if (nx.valid()) {
-        load_query<CB>(p, nx.u, t_row + kColQ, qrope, rank, h, th);
+        load_query<CB>(p, nx.u, t_row + kColQ, qrope, rank, h, hh);
         tmem_st_wait();
         fence_proxy_async_smem();
         tc_fence_before();
         __syncwarp();
         mbar_arrive_if(lane == 0 ? 1u : 0u, &c.q_full);
       }
+      SegEnd e;
+      e.b = ti.b;
+      e.hg = ti.hg;
+      e.whole = (seg_j0 == 0) && (sc.t + 1 == sc.pu1);
+      e.pidx = static_cast<size_t>(pair_id) + sc.u;
+      if (!(ok = pwait(&c.empty[it & 1u], (it >> 1) & 1u, c, pr, kPsEmpty, p.dev_err))) break;
+      tc_fence_after();
+      if (!(ok = epilogue<CB>(p, e, c, t_row, rank, rank == 0, q, hh, lane, m_ref, l_half, nq, pr))) break;
     }
     ++it;
-  }
-  if (ok && pending) {
-    if ((ok = pwait(&c.empty[(it - 1) & 1u], ((it - 1) >> 1) & 1u, c, pr, kPsEmpty, p.dev_err))) {
-      tc_fence_after();
-      ok = epilogue<CB>(p, pend, c, t_row, rank, owner, q, th, lane, m_ref, l_half, nq, pr);
-    }
   }
   if (!ok && lane == 0) stop_pair(c, pr);
 }
@@ -541,7 +584,7 @@ __device__ void mma_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, uint
     const uint32_t acc0 = tf.first ? 0u : 1u;
 #pragma unroll
     for (int ks = 0; ks < 8; ++ks)
-      umma_f16_ts(t_o, t_s + 64 * (ks >> 2) + 8 * (ks & 3), pv_b0 + boff + static_cast<uint64_t>((ks * 2048) >> 4),
+      umma_f16_ts(t_o, t_s + 16 * ks, pv_b0 + boff + static_cast<uint64_t>((ks * 2048) >> 4),
                   kIdPV, ks > 0 ? 1u : acc0);
     umma_commit(&c.empty[b]);
     QMLA_TRACE(3, it);
@@ -556,7 +599,7 @@ __device__ void mma_role(const Params& p, Sched sc, uint32_t sbase, Ctl& c, uint
 }
 
 template <int CB>
-__global__ void __launch_bounds__(kThreads, 1) decode_pair(const Params p) {
+__global__ void __launch_bounds__(kPairThreads, 1) decode_pair(const Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sbase = smem_u32(smem);
@@ -573,16 +616,19 @@ __global__ void __launch_bounds__(kThreads, 1) decode_pair(const Params p) {
   }
   if (threadIdx.x == 0) {
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&c.full[b], kWorkers);
+      mbar_init(&c.full[b], kDqWarps);
       mbar_init(&c.empty[b], 1);
     }
     mbar_init(&c.s_full, 1);
-    mbar_init(&c.p_full, kWorkers);
-    mbar_init(&c.q_full, kWorkers);
-    mbar_init(&c.o_free, kWorkers);
+    mbar_init(&c.p_full, kSWarps);
+    mbar_init(&c.q_full, kSWarps);
+    mbar_init(&c.o_free, kSWarps);
     mbar_init(&c.fin, 1);
-    mbar_init(&c.srecv_full, 128);  // the peer's four relaying warps, every lane
-    mbar_init(&c.precv_full, 128);  // the peer's four owning warps, every lane
+    for (int w = 0; w < kSWarps; ++w) {  // the peer's softmax warp w, every lane
+      mbar_init(&c.srecv[w], 32);
+      mbar_init(&c.precv[w], 32);
+      mbar_init(&c.precv2[w], 32);
+    }
     mbar_init(&c.done, 1);
     for (int i = 0; i < 4; ++i) mbar_init(&c.qbar[i], 2);
     c.abort = 0u;
@@ -600,13 +646,15 @@ __global__ void __launch_bounds__(kThreads, 1) decode_pair(const Params p) {
   Peer pr;
   pr.rank = rank ^ 1u;
   pr.abort = cluster_map(smem_u32(&c.abort), pr.rank);
-  if (warp == kMmaWarp && lane != 0) return;  // the MMA role is a single thread
+  if (warp == kPairMmaWarp && lane != 0) return;  // the MMA role is a single thread
   griddep_wait();  // prep (and the cache writer before it)
 
   Sched sc;
   sc.init(p.prefix, p.cta_info[pair_id], p.batch * p.n_hg, pair_id, p.grid);
-  if (warp < kWorkers) {
-    worker_role<CB>(p, sc, sbase, c, tmem, rank, pr, pair_id, warp, lane);
+  if (warp < kSWarps) {
+    softmax_role<CB>(p, sc, sbase, c, tmem, rank, pr, pair_id, warp, lane);
+  } else if (warp < kPairMmaWarp) {
+    dequant_role<CB>(p, sc, sbase, c, rank, pr, pair_id, warp - kSWarps, lane);
   } else {
     mma_role<CB>(p, sc, sbase, c, tmem, pr);
   }
@@ -641,7 +689,7 @@ cudaError_t launch_pairs(void (*kern)(Args...), unsigned clusters, size_t smem, 
                          Args... args) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(2 * clusters);
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(pairk::kPairThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
@@ -670,7 +718,7 @@ cudaError_t launch_pair_impl(Params prm, int sms, cudaStream_t stream, cudaEvent
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(2 * (sms / 2));
-    cfg.blockDim = dim3(kThreads);
+    cfg.blockDim = dim3(pairk::kPairThreads);
     cfg.dynamicSmemBytes = pairk::kSmem;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
