@@ -16,6 +16,7 @@
  *   *_protected         the same with sink4/local128 BF16 protection (App. C.5)
  *   *_c4r4              the same over the paper's own 20,480-byte INT4 page
  *   qmla_mla_decode_multi  several query tokens per sequence under the causal mask
+ *   qmla_mla_decode_pair   the same decode on pairs of CTAs (units of 128 query rows)
  *
  * Conventions for every call
  * --------------------------

@@ -107,6 +107,23 @@ def test_multi_query_host_checks(libqmla):
     assert L.qmla_mla_decode_multi(*args) == 1
 
 
+def test_pair_decode_host_checks(libqmla):
+    L = libqmla
+    fake = ctypes.c_void_p(0x10000)
+    base = [fake, 4, 4, fake, fake, 1, 1, 128, fake, 1, fake, 0.1, fake, None, fake, 1 << 30, None, None]
+    for i, bad in ((1, 3), (6, 0), (6, 9), (7, 0), (7, 129)):   # c_bits, q_tokens, heads
+        args = list(base)
+        args[i] = bad
+        assert L.qmla_mla_decode_pair(*args) == 1, (i, bad)
+    for T, H in ((1, 64), (3, 100), (1, 16)):                     # T x H not a multiple of 128
+        args = list(base)
+        args[6], args[7] = T, H
+        assert L.qmla_mla_decode_pair(*args) == 2, (T, H)
+    args = list(base)
+    args[12] = None                                               # no output
+    assert L.qmla_mla_decode_pair(*args) == 1
+
+
 def test_debug_hooks_host_checks(libqmla):
     L = libqmla
     fake = ctypes.c_void_p(0x10000)
