@@ -240,7 +240,9 @@ int qmla_mla_decode_multi(const void* pool_dev, int c_bits, int num_blocks, cons
  * the "global attention normalization" rule as in qmla_mla_decode).
  * q_tokens x heads must be a multiple of 128 (QMLA_ERR_UNSUPPORTED otherwise);
  * layouts, workspace size (qmla_decode_workspace_bytes(batch, q_tokens *
- * heads)), results and errors as qmla_mla_decode_multi with prot_dev = NULL. */
+ * heads)), results and errors as qmla_mla_decode_multi with prot_dev = NULL.
+ * A wait of this kernel that runs out (2 s) sets QMLA_DEVERR_TIMEOUT and one
+ * site bit among bits 17..27, and both CTAs of the pair leave. */
 int qmla_mla_decode_pair(const void* pool_dev, int c_bits, int num_blocks, const uint16_t* q_latent_dev,
                          const uint16_t* q_pe_dev, int batch, int q_tokens, int heads,
                          const int32_t* block_table_dev, int max_blocks, const int32_t* seq_lens_dev,
