@@ -623,6 +623,65 @@ def run_reference(args, ws_world: int, rank: int):
 TRACE_CTAS, TRACE_EVENTS, TRACE_TILES = 8, 128, 32
 
 
+def main_trace_summary(ev):
+    """Median stage lengths (cycles) of decode_main's steady tiles (2 .. n-2 of
+    each traced CTA). Event numbers as stamped in decode.cu: MMA thread 112 + k
+    QK of chunk k issued, 12 QK committed, 14 P seen, 15 PV issued; worker warp
+    0: 0 loop top, 16 scores seen, 19 P written, 17 every warp's P seen;
+    lane 0 of warp w: 88 + w last slot wait passed, 32 + w tile dequantised."""
+    import numpy as np
+
+    stages, period = {}, []
+    for c in range(ev.shape[0]):
+        n = int((ev[c, 12] > 0).sum())
+        for it in range(2, n - 1):
+            g, nx = ev[c, :, it], ev[c, :, it + 1]
+            period.append(nx[12] - g[12])
+            for name, v in (("mma: QK chunk 0 -> chunk 8 issued", g[120] - g[112]),
+                            ("mma: QK chunk 8 issued -> committed", g[12] - g[120]),
+                            ("mma: QK committed -> P seen", g[14] - g[12]),
+                            ("mma: P seen -> PV issued", g[15] - g[14]),
+                            ("mma: PV issued -> next QK chunk 0", nx[112] - g[15]),
+                            ("warp0: QK committed -> scores seen", g[16] - g[12]),
+                            ("warp0: scores seen -> P written", g[19] - g[16]),
+                            ("warp0: P written -> all P seen", g[17] - g[19]),
+                            ("warp0: all P seen -> row sums added", g[18] - g[17]),
+                            ("warp0: row sums added -> next loop top", nx[0] - g[18]),
+                            ("dequant: PV issued -> last slot wait passed (max warp)",
+                             max(nx[88 + w] for w in range(8)) - g[15]),
+                            ("dequant: PV issued -> tile dequantised (max warp)",
+                             max(nx[32 + w] for w in range(8)) - g[15])):
+                stages.setdefault(name, []).append(v)
+    # the next tile's dequantisation relative to this tile's PV start (P seen, event 14)
+    for c in range(ev.shape[0]):
+        n = int((ev[c, 12] > 0).sum())
+        for it in range(2, n - 1):
+            g, nx = ev[c, :, it], ev[c, :, it + 1]
+            t0 = g[14]
+            rel = {"mma PV block %d committed" % i: g[24 + i] - t0 for i in range(4)}
+            rel["mma PV issued"] = g[15] - t0
+            rel["mma next loop top"] = nx[1] - t0
+            for kc in range(5):
+                k = 2 * kc
+                rel["w0 chunk %d dq done" % k] = nx[105 + kc] - t0
+                rel["w0 chunk %d slot passed" % k] = nx[96 + kc] - t0
+                rel["w0 chunk %d arrived" % k] = nx[48 + kc] - t0
+            for kc in range(4):
+                k = 2 * kc + 1
+                rel["w4 chunk %d slot passed" % k] = nx[101 + kc] - t0
+                rel["w4 chunk %d arrived" % k] = nx[68 + kc] - t0
+            for k in range(9):
+                rel["mma next QK chunk %d issued" % k] = nx[112 + k] - t0
+            for name, v in rel.items():
+                stages.setdefault("t(PV start) + " + name, []).append(v)
+    if not period:
+        print("no steady tiles traced")
+        return
+    print(f"decode_main tile period (cycles, median over {len(period)} tiles): {np.median(period):.0f}")
+    for k, v in stages.items():
+        print(f"  {k:56s} {np.median(v):7.0f}")
+
+
 def run_trace(args):
     """Per-tile event timeline of the main decode kernel from the trace build
     (-DQMLA_TRACE_BUILD: clock64 stamps at pipeline events of the first eight
@@ -670,7 +729,8 @@ def run_trace(args):
     print(f"CTAs {len(live)}, wall us {(live[:, 1] - live[:, 0]).min() / 1e3:.1f} .. "
           f"{(live[:, 1] - live[:, 0]).max() / 1e3:.1f}, tiles per CTA {live[:, 3].min()} .. {live[:, 3].max()}")
     if not args.pair:
-        print(f"raw stamps saved to {args.trace} (decode_main's event numbers are in decode.cu)")
+        print(f"raw stamps saved to {args.trace}")
+        main_trace_summary(ev)
         return
     stages, period = {}, []
     for c in range(TRACE_CTAS):

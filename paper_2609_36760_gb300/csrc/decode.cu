@@ -141,11 +141,11 @@ static_assert(sizeof(Ctrl) % 16 == 0, "Ctrl size");
 template <int HG>
 struct Cfg {
   static constexpr int kQBytes = kNumChunks * HG * 128;
-  // O^T (4 HG columns), S^T (HG), row sums of P (HG), rounded up to a power of 2.
+  // O^T (4 HG columns) and S^T (HG), rounded up to a power of 2.
   // (HG = 128 is the unit of the cluster-pair kernel, which has its own
   // layout; only the prep and merge kernels are instantiated for it.)
   static constexpr uint32_t kTmemCols = HG >= 64 ? 512 : (HG == 32 ? 256 : 128);
-  static_assert(HG > 64 || 6 * HG <= static_cast<int>(kTmemCols), "TMEM columns");
+  static_assert(HG > 64 || 5 * HG <= static_cast<int>(kTmemCols), "TMEM columns");
   static constexpr int kSmem = 1024 + kNumChunks * kChunkBytes + kQBytes + (int)sizeof(Ctrl);
   static constexpr uint32_t kPRowBytes = 2 * HG;  // P^T tile row (one token, HG fp16)
 };
@@ -447,6 +447,49 @@ __device__ __forceinline__ void store_row(uint32_t chunk_base, int row, const Fe
   }
 }
 
+// store_row split around the slot wait for the decode workers: dq_regs
+// dequantises a packed row into registers before the wait, store_regs writes
+// it into the swizzled chunk after it, so that only the stores remain between
+// the slot's release and the chunk's arrival. Same arithmetic as store_row; a
+// row that is not fetched (f.ok false) has zero codes, scale and zero point,
+// so it dequantises to zeros without a branch.
+__device__ __forceinline__ void dq_regs(uint32_t (&o)[32], const Fetch& f, bool int4) {
+  const __half2 sz = *reinterpret_cast<const __half2*>(&f.sz);
+  const __half2 s2 = __half2half2(__low2half(sz));
+  const __half2 zz2 = __half2half2(__hadd(__high2half(sz), __float2half_rn(1024.0f)));
+  const uint32_t ss = *reinterpret_cast<const uint32_t*>(&s2);
+  const uint32_t zz = *reinterpret_cast<const uint32_t*>(&zz2);
+  constexpr uint32_t K = 0x64646464u;
+  const uint32_t w[8] = {f.a.x, f.a.y, f.a.z, f.a.w, f.b.x, f.b.y, f.b.z, f.b.w};
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    if (int4) {
+      const uint32_t lo = w[i] & 0x0F0F0F0Fu;
+      const uint32_t hi = (w[i] >> 4) & 0x0F0F0F0Fu;
+      o[4 * i + 0] = dq2(__byte_perm(lo, K, 0x4140), zz, ss);
+      o[4 * i + 1] = dq2(__byte_perm(hi, K, 0x4140), zz, ss);
+      o[4 * i + 2] = dq2(__byte_perm(lo, K, 0x4342), zz, ss);
+      o[4 * i + 3] = dq2(__byte_perm(hi, K, 0x4342), zz, ss);
+    } else {  // INT2: pieces 2m and 2m + 1 come from word m
+      const uint32_t x = w[i >> 1];
+      const uint32_t sel = (i & 1) ? 0x4342u : 0x4140u;
+      o[4 * i + 0] = dq2(__byte_perm(x & 0x03030303u, K, sel), zz, ss);
+      o[4 * i + 1] = dq2(__byte_perm((x >> 2) & 0x03030303u, K, sel), zz, ss);
+      o[4 * i + 2] = dq2(__byte_perm((x >> 4) & 0x03030303u, K, sel), zz, ss);
+      o[4 * i + 3] = dq2(__byte_perm((x >> 6) & 0x03030303u, K, sel), zz, ss);
+    }
+  }
+  // Pin the results here: the (volatile) slot wait that follows must not be
+  // hoisted above the arithmetic.
+#pragma unroll
+  for (int i = 0; i < 32; ++i) asm volatile("" : "+r"(o[i]));
+}
+__device__ __forceinline__ void store_regs(uint32_t chunk_base, int row, const uint32_t (&o)[32]) {
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+    sts_v4(chunk_base + swz_off(row, i, 128), o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
+}
+
 // Rows of the paper's page. store_row_c4r4 writes one row (64 INT4 codes) of
 // chunk k as RN_f16(s (q - z)) with the stored bf16 (content) or fp32 (RoPE)
 // scale. q - z is exact in fp16 (as in store_row); a bf16 scale in [2^-14,
@@ -711,28 +754,21 @@ struct SegEnd {
   size_t pidx;  // partial slot (CTA index + unit)
 };
 
-// Segment end: l[h] = sum of the row sums, then out = O / l (or the partial
-// o, m, l) for this warp's heads, then release O^T to the next segment.
+// Segment end: l[h] = sum of the four row quarters' sums, then out = O / l
+// (or the partial o, m, l) for this warp's heads, then release O^T to the next
+// segment. lsum[c] holds, in the lanes that warp_colsum leaves it in, this
+// warp's sum over its 32 rows and the segment's tiles of head column group c.
 template <int CB, int HG>
-__device__ bool epilogue(const Params& p, const SegEnd& e, Ctrl& ctl, uint32_t tmem, uint32_t& gph, int warp,
-                         int lane) {
+__device__ bool epilogue(const Params& p, const SegEnd& e, Ctrl& ctl, uint32_t tmem, uint32_t& gph,
+                         const float (&lsum)[Cols<HG>::kN], int warp, int lane) {
   using C = Cols<HG>;
   const int q4 = warp & 3, half = warp >> 2, row = q4 * 32 + lane, cb0 = half * C::kPerWarp;
   const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
-  const uint32_t t_l = tmem + 5 * HG + cb0 + lane_off;
   const uint32_t t_o = tmem + cb0 + lane_off;
+  constexpr int kSh = C::kW == 16 ? 1 : 2;
 #pragma unroll
-  for (int c = 0; c < C::kN; ++c) {
-    uint32_t r[C::kW];
-    tmem_ld(t_l + c * C::kW, r);
-    tmem_ld_wait();
-    float v[C::kW];
-#pragma unroll
-    for (int jj = 0; jj < C::kW; ++jj) v[jj] = __uint_as_float(r[jj]);
-    const float tot = warp_colsum<C::kW>(v, lane);
-    constexpr int kSh = C::kW == 16 ? 1 : 2;
-    if ((lane & ((1 << kSh) - 1)) == 0) ctl.red[q4][cb0 + c * C::kW + (lane >> kSh)] = tot;
-  }
+  for (int c = 0; c < C::kN; ++c)
+    if ((lane & ((1 << kSh) - 1)) == 0) ctl.red[q4][cb0 + c * C::kW + (lane >> kSh)] = lsum[c];
   if (!group_sync(ctl, gph, p.dev_err)) return false;
   const int tid = threadIdx.x;  // 0 .. 255 over the worker warps
   if (tid < HG) {
@@ -826,7 +862,6 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
   const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
   const uint32_t t_s = tmem + 4 * HG + cb0 + lane_off;
   const uint32_t t_o = tmem + cb0 + lane_off;
-  const uint32_t t_l = tmem + 5 * HG + cb0 + lane_off;
   const uint32_t ptile = chunks + 8 * kChunkBytes;
   const float sl2 = p.scale_log2;
   constexpr int kMyChunks = 5;  // chunks per parity, rounded up (parity 1 has 4)
@@ -835,6 +870,11 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
   bool ok = true;
   bool pending = false;  // the previous tile ended a segment whose epilogue is still due
   SegEnd pend{};
+  // Row sums of P for the current segment: per head column group, the warp's
+  // column sum over its 32 rows (warp_colsum layout), accumulated over tiles.
+  float lsum[C::kN], lsum_done[C::kN];  // lsum_done: the pending segment's sums
+#pragma unroll
+  for (int c = 0; c < C::kN; ++c) lsum[c] = lsum_done[c] = 0.0f;
 
   // Packed rows of the tile about to be dequantised (INT4/INT2), fetched a tile ahead.
   Fetch f[kMyChunks];
@@ -897,12 +937,18 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     if (lane == 0 && warp == 0) QMLA_TRACE(0, it);
 
     // ---- dequantise this tile, chunk by chunk as the previous PV frees the slots
+    // (this library's INT4 / INT2 block: the arithmetic before the slot wait)
+    constexpr bool kEarly = (CB == 4 || CB == 2) && !PROT;
 #pragma unroll
     for (int kc = 0; kc < kMyChunks; ++kc) {
       const int k = 2 * kc + par;
       if (k >= kNumChunks) break;
+      uint32_t dq[kEarly ? 32 : 1];
+      if constexpr (kEarly) dq_regs(dq, f[kc], CB == 4 || k == 8);
+      if (lane == 0 && warp == 0) QMLA_TRACE(105 + kc, it);
       if (!(ok = wwait(slot_bar(ctl, k), (it & 1u) ^ 1u, ctl, kSiteDqSlot, p.dev_err))) break;
       if (lane == 0) QMLA_TRACE(88 + warp, it);  // (overwritten per chunk: last slot wait)
+      if (lane == 0 && (warp & 3) == 0) QMLA_TRACE((warp == 0 ? 96 : 101) + kc, it);
       if constexpr (CB == 16) {
         uint4 nxt[8];
         const int kn = k + 2;
@@ -919,12 +965,18 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
 #pragma unroll
         for (int i = 0; i < 8; ++i) cur[i] = nxt[i];
       } else {
-        dq_row<CB, PROT>(chunks + k * kChunkBytes, row, k, psrc_cur, f[kc]);
-        f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);  // the next tile's rows of this chunk
+        if constexpr (kEarly) {
+          store_regs(chunks + k * kChunkBytes, row, dq);
+        } else {
+          dq_row<CB, PROT>(chunks + k * kChunkBytes, row, k, psrc_cur, f[kc]);
+          f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);  // the next tile's rows of this chunk
+        }
       }
       fence_proxy_async_smem();
       __syncwarp();
       mbar_arrive_if(lane == 0 ? 1u : 0u, &ctl.chunk_full[k]);
+      // (the early path fetches the next tile's rows of this chunk after the arrive)
+      if constexpr (kEarly) f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);
       if (lane == 0) QMLA_TRACE(48 + warp * 5 + kc, it);
     }
     if (!ok) break;
@@ -934,13 +986,13 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     psrc_cur = psrc_nx;
     nx = nn;
     ref_nx = ref_nn;
-    const TileInfo ti = tile_info(sc, p);  // ntok of this tile for the softmax (loaded long ago)
+    const TileInfo ti = tile_info(sc, p);  // ntok of this tile for the softmax
     const int lim = row_limit<HG>(p, ti, row, cb0);
 
     // ---- the previous segment's results (its last PV completed: chunks 6..8 were waited for)
     if (pending) {
       tc_fence_after();
-      if (!(ok = epilogue<CB, HG>(p, pend, ctl, tmem, gph, warp, lane))) break;
+      if (!(ok = epilogue<CB, HG>(p, pend, ctl, tmem, gph, lsum_done, warp, lane))) break;
       pending = false;
       if (lane == 0 && warp == 0) QMLA_TRACE(20, it);
     }
@@ -990,9 +1042,12 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       }
       if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
       if (!ti.first) {
+        constexpr int kSh = C::kW == 16 ? 1 : 2;
 #pragma unroll
-        for (int i = 0; i < 5; ++i) {  // O^T blocks 0..3 and the row sums (column block 5)
-          const uint32_t col = i < 4 ? i * HG : 5 * HG;
+        for (int c = 0; c < C::kN; ++c) lsum[c] *= ctl.alpha[cb0 + c * C::kW + (lane >> kSh)];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {  // O^T blocks 0..3
+          const uint32_t col = i * HG;
 #pragma unroll
           for (int c = 0; c < C::kN; ++c) {
             uint32_t r[C::kW];
@@ -1013,24 +1068,24 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       mbar_arrive_if(lane == 0 ? 1u : 0u, &ctl.p_fixed);
       ++nresc;
     }
-    // Row sums of the fp16 weights the PV MMA multiplies with (no MMA reads them).
+    // Row sums of the fp16 weights the PV MMA multiplies with: this warp's column
+    // sums over its 32 rows, added to the segment's running sums in registers.
 #pragma unroll
     for (int c = 0; c < C::kN; ++c) {
-      uint32_t r[C::kW];
-      if (!ti.first) {
-        tmem_ld(t_l + c * C::kW, r);
-        tmem_ld_wait();
-      }
+      float v[C::kW];
 #pragma unroll
       for (int jj = 0; jj < C::kW; jj += 2) {
         const float2 pf = __half22float2(*reinterpret_cast<const __half2*>(&pk[c * (C::kW / 2) + (jj >> 1)]));
-        r[jj] = __float_as_uint(ti.first ? pf.x : __uint_as_float(r[jj]) + pf.x);
-        r[jj + 1] = __float_as_uint(ti.first ? pf.y : __uint_as_float(r[jj + 1]) + pf.y);
+        v[jj] = pf.x;
+        v[jj + 1] = pf.y;
       }
-      tmem_st(t_l + c * C::kW, r);
+      const float t = warp_colsum<C::kW>(v, lane);
+      lsum[c] = ti.first ? t : lsum[c] + t;
     }
-    tmem_st_wait();
+    if (lane == 0 && warp == 0) QMLA_TRACE(18, it);
     if (ti.last) {
+#pragma unroll
+      for (int c = 0; c < C::kN; ++c) lsum_done[c] = lsum[c];
       pending = true;
       pend.b = ti.b;
       pend.hg = ti.hg;
@@ -1043,7 +1098,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
   if (ok && pending) {
     if ((ok = wwait(&ctl.pv_done, (it - 1) & 1u, ctl, kSitePvEpi, p.dev_err))) {
       tc_fence_after();
-      ok = epilogue<CB, HG>(p, pend, ctl, tmem, gph, warp, lane);
+      ok = epilogue<CB, HG>(p, pend, ctl, tmem, gph, lsum_done, warp, lane);
     }
   }
   if (!ok && lane == 0) set_abort(ctl, p.dev_err);
@@ -1093,6 +1148,7 @@ __device__ void mma_thread(const Params& p, Sched sc, uint32_t chunks, uint8_t* 
   if (sc.valid()) issue_query<HG>(p, sc.u, qsmem, ctl);
   for (; ok && sc.valid(); sc.next()) {
     const TileFlags ti = tile_flags(sc);
+    QMLA_TRACE(1, it);
     if (ti.first && !(ok = twait(&ctl.q_full, seg & 1u, ctl, kSiteMmaQFull, p.dev_err))) break;
     // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576), chunk by
     // chunk. The next chunk's barrier is probed before this chunk's MMAs are
@@ -1139,6 +1195,7 @@ __device__ void mma_thread(const Params& p, Sched sc, uint32_t chunks, uint8_t* 
         umma_f16_ss(tmem + i * HG, pv_a0 + static_cast<uint64_t>((2 * i * kChunkBytes + kk * 2048) >> 4),
                     pv_b0 + static_cast<uint64_t>((kk * 2 * kSboP) >> 4), kIdPV, kk == 0 ? acc0 : 1u);
       umma_commit(i < 3 ? &ctl.slot_free[i] : &ctl.pv_done);
+      QMLA_TRACE(24 + i, it);
     }
     QMLA_TRACE(15, it);
     ++it;
