@@ -2,10 +2,13 @@
 """Benchmark of the low-bit MLA decode hot path on GB300.
 
 One step = qmla_quant_append of one new token per sequence followed by
-qmla_mla_decode over every cached token (plan + main + combine kernels), on
+qmla_mla_decode over every cached token (plan, main and merge kernels), on
 the DeepSeek-V3-shaped workload (64 sequences x 128 heads, 4096 cached tokens
 plus the appended one, INT4 content + INT4 RoPE key) unless --workload says
 otherwise. The metric is KV-tokens/s: tokens attended per step / step time.
+The default run then measures the other workloads the same way and reports
+them under "configs" (the 128-sequence serving mix over its 256 steps, also on
+the BF16 comparison cache, and the DeepSeek-V3 workload on the BF16 cache).
 
 Contract: `python bench.py --gpus N --steps K --warmup W` prints one JSON line
 (rank 0). With N > 1 (torchrun) every rank decodes its own copy of the
@@ -55,9 +58,8 @@ def parse(argv=None):
     ap.add_argument("--q-tokens", type=int, default=1,
                     help="query tokens per sequence (multi-token prediction / speculative verification); each step "
                          "appends that many tokens and scores them under the causal mask")
-    ap.add_argument("--pair", action="store_true",
-                    help="decode on CTA pairs (qmla_mla_decode_pair; heads x q-tokens a multiple of 128, "
-                         "INT4/INT2 block, no protection)")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the other workloads (configs) measured after the headline one")
     ap.add_argument("--trace", default=None, metavar="NPZ",
                     help="instead of timing: build the trace library, trace one decode step's main kernel, print "
                          "the per-tile stage breakdown and save the raw clock64 stamps to NPZ")
@@ -188,13 +190,12 @@ class Workspace:
     """GPU state of one workload: pool, block table, per-step inputs."""
 
     def __init__(self, w: W.Workload, bf16: bool, dev: torch.device, nsteps: int, protect: bool = False,
-                 c4r4: bool = False, q_tokens: int = 1, pair: bool = False):
+                 c4r4: bool = False, q_tokens: int = 1, gen_device=None):
+        """gen_device None draws the inputs with the host generators (the values the
+        oracle sees); a CUDA device draws them there (same distributions)."""
         import paper_2609_36760_gb300 as Q
         self.Q = Q
         self.q_tokens = q_tokens
-        self.pair = pair
-        if pair and (bf16 or c4r4 or protect or (q_tokens * w.heads) % 128 != 0):
-            raise SystemExit("--pair decodes the INT4/INT2 block without protection, heads x q-tokens % 128 == 0")
         if q_tokens > 1:
             if bf16 or c4r4:
                 raise SystemExit("--q-tokens > 1 runs on the INT4/INT2 block (protection optional)")
@@ -219,8 +220,8 @@ class Workspace:
         # Prefill through the library, one sequence at a time (bounded host memory).
         for b in range(w.batch):
             n_all = self.prefill[b] + w.append * self.nsteps
-            lat = W.latent_for_seq(w, b, n_all, gains)
-            kp = W.kpe_for_seq(w, b, n_all)
+            lat = W.latent_for_seq(w, b, n_all, gains, device=gen_device)
+            kp = W.kpe_for_seq(w, b, n_all, device=gen_device)
             n = self.prefill[b]
             self._append(lat[:n].to(dev), kp[:n].to(dev), torch.full((n,), b, dtype=torch.int32, device=dev),
                          torch.arange(n, dtype=torch.int32, device=dev), self.prefill_lens)
@@ -234,7 +235,7 @@ class Workspace:
         self.steps = []
         for s in range(self.nsteps):
             si = self.step_in[s]
-            ql, qp = W.queries(w, s) if q_tokens == 1 else W.queries_multi(w, s, q_tokens)
+            ql, qp = W.queries(w, s, device=gen_device) if q_tokens == 1 else W.queries_multi(w, s, q_tokens)
             lens = [n + w.append * (s + 1) for n in self.prefill]
             host = {
                 "lat": torch.cat(si["lat"]) if si["lat"] else torch.zeros(0, 512, dtype=torch.bfloat16),
@@ -244,6 +245,8 @@ class Workspace:
                 "ql": ql.contiguous(), "qp": qp.contiguous(),
                 "lens": torch.tensor(lens, dtype=torch.int32),
             }
+            if gen_device is not None:
+                host = {k: v.cpu() for k, v in host.items()}
             self.steps.append({"host": host, "dev": {k: v.to(dev) for k, v in host.items()}, "lens": lens})
         qshape = (w.batch, w.heads) if q_tokens == 1 else (w.batch, q_tokens, w.heads)
         self.out = torch.empty(qshape + (512,), dtype=torch.float32, device=dev)
@@ -271,10 +274,16 @@ class Workspace:
         self._append(d["lat"], d["kp"], d["sid"], d["pos"], d["lens"])
         self.decode(d, out, lse)
 
-    def decode(self, d: dict, out, lse):
-        if self.pair:
-            self.Q.mla_decode_pair(self.pool, self.w.c_bits, d["ql"], d["qp"], self.table, d["lens"], TAU, out, lse,
-                                   self.ws, self.err)
+    def cache_kind(self):
+        return "bf16" if self.bf16 else ("c4r4" if self.c4r4 else self.w.c_bits)
+
+    def decode(self, d: dict, out, lse, events=None):
+        """One decode call through the variant's own entry point; with events
+        (before, after) through qmla_mla_decode_ex, which records them around the
+        main kernel of this call."""
+        if events is not None:
+            self.Q.mla_decode_ex(self.pool, self.cache_kind(), d["ql"], d["qp"], self.table, d["lens"], TAU, out,
+                                 lse, self.ws, self.err, prot=self.prot, events=events)
         elif self.q_tokens > 1:
             self.Q.mla_decode_multi(self.pool, self.w.c_bits, d["ql"], d["qp"], self.table, d["lens"], TAU, out,
                                     lse, self.ws, self.err, prot=self.prot)
@@ -295,48 +304,34 @@ class Workspace:
         return (1 if self.w.append > 0 else 0) + 3
 
 
-def run_native(args, ws_world: int, rank: int, local: int):
-    import paper_2609_36760_gb300 as Q
-    dev = torch.device("cuda", local)
-    torch.cuda.set_device(dev)
-    Q.lib()
-    dist = None
-    if ws_world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=dev)
-    w = W.WORKLOADS[args.workload]
-    K, Wm = args.steps, args.warmup
-    state = Workspace(w, args.bf16_cache, dev, K + Wm, protect=args.protect, c4r4=args.c4r4, q_tokens=args.q_tokens,
-                      pair=args.pair)
-    w = state.w
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # larger than the 126 MB L2
+def time_steps(state: Workspace, K: int, Wm: int, flush, dev, clocks=None, dist=None):
+    """Warm-up, then pass A (K whole steps as a user runs them: the library's
+    launches overlap their start-up; CUDA events around each step) and pass B
+    (min(K, 100) steps whose main decode kernel is bracketed by per-call events,
+    which make the call's launches wait for one another in full). The L2 is
+    flushed (256 MB write) before every step of both passes."""
+    Q = state.Q
     stream = torch.cuda.current_stream(dev)
-
-    # warm-up (untimed)
     for i in range(Wm):
         flush.zero_()
         state.step(i)
     torch.cuda.synchronize(dev)
     if Q.read_dev_err(state.err) != 0:
         raise RuntimeError(f"device error word {Q.read_dev_err(state.err):#x} after warm-up")
-
-    # Pass A times whole steps as a user runs them (value); pass B brackets the
-    # main kernel with events (roofline). Events between the library's launches
-    # make each launch wait for the previous one in full, so pass A sets none.
     Km = min(K, 100)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
-    # pass B events: before the append, after it, around the main kernel (set in the library), after the merge
+    # pass B events: before the append, after it, around the main kernel (recorded by the library), after the call
     evm = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(Km)]
     for e in ev + evm:
         for x in e:
             x.record(stream)
     torch.cuda.synchronize(dev)
-    clocks = ClockSampler(local)
     if dist is not None:
         dist.barrier()
     torch.cuda.synchronize(dev)
-    clocks.start()
-    time.sleep(0.15)
+    if clocks is not None:
+        clocks.start()
+        time.sleep(0.15)
     t_wall0 = time.perf_counter()
     for i in range(K):
         e0, e1 = ev[i]
@@ -349,48 +344,42 @@ def run_native(args, ws_world: int, rank: int, local: int):
     for i in range(Km):
         a0, a1, m0, m1, e_end = evm[i]
         flush.zero_()
-        Q.set_profile_events(m0, m1)
         d = state.steps[(Wm + i) % state.nsteps]["dev"]
         a0.record(stream)
         state._append(d["lat"], d["kp"], d["sid"], d["pos"], d["lens"])  # the same appends again: cache unchanged
         a1.record(stream)
-        state.decode(d, state.out, state.lse)
+        state.decode(d, state.out, state.lse, events=(m0, m1))
         e_end.record(stream)
     torch.cuda.synchronize(dev)
-    Q.set_profile_events(None, None)
     if dist is not None:
         dist.barrier()
     torch.cuda.synchronize(dev)
-    clk = clocks.stop()
+    clk = clocks.stop() if clocks is not None else None
     err = Q.read_dev_err(state.err)
     if err != 0:
         raise RuntimeError(f"device error word {err:#x} in the timed loop")
-
-    step_ms = [ev[i][0].elapsed_time(ev[i][1]) for i in range(K)]
-    main_ms = [evm[i][2].elapsed_time(evm[i][3]) for i in range(Km)]
     med = lambda xs: statistics.median(xs) * 1e3  # noqa: E731
     parts_us = {"append": round(med([e[0].elapsed_time(e[1]) for e in evm]), 2),
                 "prep_and_gaps": round(med([e[1].elapsed_time(e[2]) for e in evm]), 2),
-                "main": round(med(main_ms), 2),
+                "main": round(med([e[2].elapsed_time(e[3]) for e in evm]), 2),
                 "merge_and_gap": round(med([e[3].elapsed_time(e[4]) for e in evm]), 2),
                 "note": "medians of pass B, whose events serialise the launches"}
-    qs = statistics.quantiles(step_ms, n=10) if K >= 10 else [min(step_ms)] * 9
-    step_dist_us = {"median": round(med(step_ms), 2), "p10": round(qs[0] * 1e3, 2), "p90": round(qs[-1] * 1e3, 2)}
-    ms_step = sum(step_ms) / K
-    ms_main = sum(main_ms) / Km
-    ms_step_max = max_over_ranks(ms_step, dist, dev)
-
+    step_ms = [ev[i][0].elapsed_time(ev[i][1]) for i in range(K)]
+    main_ms = [evm[i][2].elapsed_time(evm[i][3]) for i in range(Km)]
     lens_all = [state.steps[(Wm + i) % state.nsteps]["lens"] for i in range(K)]
-    tok_per_step = sum(sum(l) for l in lens_all) / K
-    value = whole_job_value(ws_world, tok_per_step, ms_step_max)
+    return {"step_ms": step_ms, "main_ms": main_ms, "parts_us": parts_us, "clocks": clk, "wall_s": t_wall,
+            "tokens_per_step": sum(sum(l) for l in lens_all) / K, "lens0": lens_all[0]}
 
-    # roofline of the main decode kernel
+
+def roofline(w: W.Workload, lens, bf16: bool, c4r4: bool, q_tokens: int, ms_main: float):
+    """Roofline of the main decode kernel: the slower of algorithmic FLOPs over
+    the measured bf16 tensor peak and algorithmic bytes over the measured HBM
+    copy bandwidth; achieved = the bound's quantity / the kernel's event time."""
     peaks, peak_src = load_peaks()
-    flops, nbytes = workload_cost(w, lens_all[0], args.bf16_cache, state.c4r4, args.q_tokens)
+    flops, nbytes = workload_cost(w, lens, bf16, c4r4, q_tokens)
     t_tc = flops / (peaks["bf16_tflops"] * 1e12)
     t_hbm = nbytes / (peaks["hbm_gbs"] * 1e9)
-    tensor_bound = t_tc >= t_hbm
-    if tensor_bound:
+    if t_tc >= t_hbm:
         achieved = flops / (ms_main * 1e-3) / 1e12
         roof = {"bound": "tensor", "achieved": round(achieved, 2), "peak": peaks["bf16_tflops"], "unit": "TFLOP/s"}
     else:
@@ -398,18 +387,47 @@ def run_native(args, ws_world: int, rank: int, local: int):
         roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s"}
     roof["frac"] = round(achieved / roof["peak"], 4)
     roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
+    roof["kernel_us"] = round(ms_main * 1e3, 2)
+    roof["algorithmic_flops"] = flops
+    roof["algorithmic_bytes"] = nbytes
+    roof["roofline_us"] = round(max(t_tc, t_hbm) * 1e6, 2)
+    return roof
+
+
+def run_native(args, ws_world: int, rank: int, local: int):
+    import paper_2609_36760_gb300 as Q
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    Q.lib()
+    dist = None
+    if ws_world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    w = W.WORKLOADS[args.workload]
+    K, Wm = args.steps, args.warmup
+    state = Workspace(w, args.bf16_cache, dev, K + Wm, protect=args.protect, c4r4=args.c4r4, q_tokens=args.q_tokens)
+    w = state.w
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # larger than the 126 MB L2
+    t = time_steps(state, K, Wm, flush, dev, clocks=ClockSampler(local), dist=dist)
+    step_ms, main_ms = t["step_ms"], t["main_ms"]
+    med = lambda xs: statistics.median(xs) * 1e3  # noqa: E731
+    qs = statistics.quantiles(step_ms, n=10) if K >= 10 else [min(step_ms)] * 9
+    step_dist_us = {"median": round(med(step_ms), 2), "p10": round(qs[0] * 1e3, 2), "p90": round(qs[-1] * 1e3, 2)}
+    ms_step_max = max_over_ranks(sum(step_ms) / K, dist, dev)
+    ms_main = sum(main_ms) / len(main_ms)
+    tok_per_step = t["tokens_per_step"]
+    value = whole_job_value(ws_world, tok_per_step, ms_step_max)
+
+    roof = roofline(w, t["lens0"], args.bf16_cache, state.c4r4, args.q_tokens, ms_main)
     prof = profile_traffic(decode_cu_hash())
     roof["traffic"] = (prof["dram_bytes_per_launch"] if prof and prof.get("workload") == args.workload
                        and bool(prof.get("bf16_cache")) == bool(args.bf16_cache)
                        and bool(prof.get("protect")) == bool(args.protect)
                        and bool(prof.get("c4r4")) == bool(state.c4r4)
-                       and int(prof.get("q_tokens", 1)) == args.q_tokens
-                       and bool(prof.get("pair")) == bool(args.pair) else None)
-    roof["kernel"] = "decode_pair" if args.pair else "decode_main"
-    roof["kernel_us"] = round(ms_main * 1e3, 2)
-    roof["algorithmic_flops"] = flops
-    roof["algorithmic_bytes"] = nbytes
-    roof["roofline_us"] = round(max(t_tc, t_hbm) * 1e6, 2)
+                       and int(prof.get("q_tokens", 1)) == args.q_tokens else None)
+    if roof["traffic"] is not None:
+        roof["traffic_source"] = prof.get("source", "profiles/decode_main_traffic.json")
+    roof["kernel"] = "decode_main"
 
     # end to end through the public API with host buffers
     e2e = None
@@ -422,27 +440,94 @@ def run_native(args, ws_world: int, rank: int, local: int):
         "dtype": "f16", "data": "synthetic (seeded generators, workloads/synthetic.py)",
         "config": {"workload": w.name, "batch_per_gpu": w.batch, "heads": w.heads, "c_bits": w.c_bits,
                    "pe_bits": 4, "cache": cache_name(w, args.bf16_cache, args.protect, state.c4r4),
-                   "q_tokens_per_seq": args.q_tokens,
-                   "kernel": "CTA pairs (qmla_mla_decode_pair)" if args.pair else "one CTA per SM (qmla_mla_decode)",
+                   "q_tokens_per_seq": args.q_tokens, "kernel": "one CTA per SM (qmla_mla_decode)",
                    "kv_tokens_per_step_per_gpu": tok_per_step, "l2": "flushed (256 MB write) before every timed step",
                    "parallelism": f"replicas x{ws_world} (independent sequences)"},
         "us_per_step": round(ms_step_max * 1e3, 2),
         "us_per_step_dist": step_dist_us,
-        "step_parts_us": parts_us,
+        "step_parts_us": t["parts_us"],
         "roofline": roof,
         "gpu_launches": state.launches_per_step() * K,
-        "clocks": clk,
+        "clocks": t["clocks"],
         "e2e": e2e,
-        "wall_s_timed_loop": round(t_wall, 3),
+        "wall_s_timed_loop": round(t["wall_s"], 3),
     }
     if rank == 0 and ws_world == 1 and not args.no_cpu_baseline:
         res["cpu_baseline"] = cpu_baseline(w, args.bf16_cache, budget_s=15.0, protect=args.protect,
                                            c4r4=state.c4r4, q_tokens=args.q_tokens)
+    if ws_world == 1 and not args.no_configs and args.workload == DEFAULT_WORKLOAD and not (
+            args.bf16_cache or args.protect or args.c4r4 or args.q_tokens != 1):
+        del state
+        torch.cuda.empty_cache()
+        res["configs"] = run_configs(dev, flush, K)
+        b16 = res["configs"].get(w.name + "_bf16cache")
+        if b16 is not None:  # INT4 (this line) against the same kernel on the BF16 cache
+            b16["int4_speedup_step"] = round(b16["us_per_step"] / res["us_per_step"], 3)
+            b16["int4_speedup_main"] = round(b16["roofline"]["kernel_us"] / roof["kernel_us"], 3)
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
     if rank == 0:
         print(json.dumps(res), flush=True)
+
+
+# The other workloads measured after the headline one (one line per config):
+# (workload, BF16 comparison cache). Their inputs are drawn on the GPU with the
+# same seeded distributions (the host generators would take minutes for the
+# 1M-token workloads); the headline workload keeps the host generators, whose
+# values the oracle baseline uses.
+CONFIGS = [("tiny_b1_h16_l256_int4", False), ("int2_b32_h128_l32768", False), ("long_b4_h64_l128k", False),
+           ("serve_b128_h16_mix", False), ("serve_b128_h16_mix", True), ("dsv3_b64_h128_l4096_int4", True)]
+
+
+def run_configs(dev, flush, K: int) -> dict:
+    """Every other workload, each timed like the headline one (time_steps): step
+    time, KV-tokens/s and the main kernel's roofline fraction. The serving mix
+    runs its 256 consecutive steps (append 1 token per sequence + decode), on
+    the INT4 cache and on the BF16 comparison cache; the 128K workload adds the
+    physical cache bytes of a 128K-token sequence against a BF16 cache."""
+    import paper_2609_36760_gb300 as Q
+    out = {}
+    for name, bf16 in CONFIGS:
+        w = W.WORKLOADS[name]
+        Kc, Wc = (w.steps, 3) if w.steps > 1 else (min(K, 20), 3)
+        state = Workspace(w, bf16, dev, Kc + Wc, gen_device=dev)
+        t = time_steps(state, Kc, Wc, flush, dev)
+        step_ms, main_ms = t["step_ms"], t["main_ms"]
+        ms_step = sum(step_ms) / len(step_ms)
+        ms_main = sum(main_ms) / len(main_ms)
+        roof = roofline(state.w, t["lens0"], bf16, False, 1, ms_main)
+        qs = statistics.quantiles(step_ms, n=10) if len(step_ms) >= 10 else [min(step_ms)] * 9
+        r = {"cache": cache_name(w, bf16, False, False), "batch": w.batch, "heads": w.heads,
+             "steps": Kc, "warmup": Wc, "us_per_step": round(ms_step * 1e3, 2),
+             "us_per_step_dist": {"median": round(statistics.median(step_ms) * 1e3, 2),
+                                  "p10": round(qs[0] * 1e3, 2), "p90": round(qs[-1] * 1e3, 2)},
+             "kv_tokens_per_s": round(t["tokens_per_step"] / (ms_step * 1e-3), 1),
+             "kv_tokens_per_step": t["tokens_per_step"], "step_parts_us": t["parts_us"],
+             "roofline": {k: roof[k] for k in ("bound", "achieved", "peak", "unit", "frac", "kernel_us",
+                                              "roofline_us", "algorithmic_bytes", "algorithmic_flops")},
+             "hbm_gbs_of_step": round(roof["algorithmic_bytes"] / (ms_step * 1e-3) / 1e9, 1),
+             "gpu_launches": state.launches_per_step() * Kc,
+             "inputs": "seeded, drawn on the GPU (same distributions as workloads/synthetic.py)"}
+        if name == "long_b4_h64_l128k":
+            blocks = (131072 + 63) // 64
+            r["physical_cache_bytes_128k"] = {
+                "int4_int4_block": blocks * Q.block_bytes(4), "bf16": blocks * Q.bf16_block_bytes(),
+                "ratio": round(Q.bf16_block_bytes() / Q.block_bytes(4), 3),
+                "paper_ratio_context": 3.59,
+                "note": "values + fp16 scales + fp16 zeros of one 131072-token sequence, no protection buffer"}
+        out[name + ("_bf16cache" if bf16 else "")] = r
+        del state
+        torch.cuda.empty_cache()
+    for base in ("serve_b128_h16_mix", "dsv3_b64_h128_l4096_int4"):
+        b16 = out.get(base + "_bf16cache")
+        i4 = out.get(base)
+        if b16 is not None:
+            if i4 is None:  # the headline workload's INT4 figures are the line's own
+                continue
+            b16["int4_speedup_step"] = round(b16["us_per_step"] / i4["us_per_step"], 3)
+            b16["int4_speedup_main"] = round(b16["roofline"]["kernel_us"] / i4["roofline"]["kernel_us"], 3)
+    return out
 
 
 def cache_name(w: W.Workload, bf16: bool, protect: bool, c4r4: bool) -> str:
@@ -686,13 +771,8 @@ def run_trace(args):
     """Per-tile event timeline of the main decode kernel from the trace build
     (-DQMLA_TRACE_BUILD: clock64 stamps at pipeline events of the first eight
     CTAs, written through the buffer given to qmla_trace_set). Stamps are per-SM
-    clocks: only differences within one CTA mean anything. Events of the
-    CTA-pair kernel: MMA thread 0 loop top, 4 QK issued, 1 QK committed, 2 P
-    seen, 3 PV committed; lane 0 of softmax warps 0 and 2 at 8 + k and 16 + k,
-    k = 0 loop top, 3 scores seen, 4 relayed scores sent and own scores read,
-    5 peer scores added and the tile max agreed in the CTA, 6 P and max sent,
-    7 P in TMEM (after the peer's P, and a second exchange when the reference
-    moved)."""
+    clocks: only differences within one CTA mean anything (event numbers in
+    main_trace_summary)."""
     import ctypes
 
     import numpy as np
@@ -708,7 +788,7 @@ def run_trace(args):
     L.qmla_trace_set.argtypes, L.qmla_trace_set.restype = [ctypes.c_void_p], ctypes.c_int
     dev = torch.device("cuda", 0)
     st = Workspace(W.WORKLOADS[args.workload], args.bf16_cache, dev, 4, protect=args.protect, c4r4=args.c4r4,
-                   q_tokens=args.q_tokens, pair=args.pair)
+                   q_tokens=args.q_tokens)
     buf = torch.zeros(TRACE_CTAS * TRACE_EVENTS * TRACE_TILES + 4 * 1024, dtype=torch.int64, device=dev)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     for i in range(3):
@@ -728,29 +808,8 @@ def run_trace(args):
     live = cta[cta[:, 0] > 0]
     print(f"CTAs {len(live)}, wall us {(live[:, 1] - live[:, 0]).min() / 1e3:.1f} .. "
           f"{(live[:, 1] - live[:, 0]).max() / 1e3:.1f}, tiles per CTA {live[:, 3].min()} .. {live[:, 3].max()}")
-    if not args.pair:
-        print(f"raw stamps saved to {args.trace}")
-        main_trace_summary(ev)
-        return
-    stages, period = {}, []
-    for c in range(TRACE_CTAS):
-        n = int((ev[c, 0] > 0).sum())
-        period += list(np.diff(ev[c, 0, :n])[2:])
-        for it in range(2, n - 1):
-            g = ev[c, :, it]
-            for name, v in (("mma: loop top -> QK issued", g[4] - g[0]), ("mma: QK committed -> P seen", g[2] - g[1]),
-                            ("mma: P seen -> PV committed", g[3] - g[2])):
-                stages.setdefault(name, []).append(v)
-            for w0 in (8, 16):
-                for name, v in (("softmax: loop top -> scores seen", g[w0 + 3] - g[w0]),
-                                ("softmax: relay sent, own read", g[w0 + 4] - g[w0 + 3]),
-                                ("softmax: peer scores, max agreed", g[w0 + 5] - g[w0 + 4]),
-                                ("softmax: P and max sent", g[w0 + 6] - g[w0 + 5]),
-                                ("softmax: peer P, P in TMEM", g[w0 + 7] - g[w0 + 6])):
-                    stages.setdefault(name, []).append(v)
-    print(f"tile period (cycles, median): {np.median(period):.0f}")
-    for k, v in stages.items():
-        print(f"  {k:36s} {np.median(v):7.0f}")
+    print(f"raw stamps saved to {args.trace}")
+    main_trace_summary(ev)
 
 
 def main():

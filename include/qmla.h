@@ -16,7 +16,8 @@
  *   *_protected         the same with sink4/local128 BF16 protection (App. C.5)
  *   *_c4r4              the same over the paper's own 20,480-byte INT4 page
  *   qmla_mla_decode_multi  several query tokens per sequence under the causal mask
- *   qmla_mla_decode_pair   the same decode on pairs of CTAs (units of 128 query rows)
+ *   qmla_mla_decode_ex  every decode variant from one descriptor, with optional
+ *                       per-call events around the main kernel
  *
  * Conventions for every call
  * --------------------------
@@ -230,25 +231,6 @@ int qmla_mla_decode_multi(const void* pool_dev, int c_bits, int num_blocks, cons
                           void* workspace_dev, size_t workspace_bytes, uint32_t* dev_err_dev,
                           qmla_stream_t stream);
 
-/* qmla_mla_decode_multi (INT4 / INT2 block, no protection) on pairs of CTAs
- * (thread-block clusters of two): each unit of 128 query rows of a sequence is
- * computed by two SMs, each holding half of the 576 channels of every
- * reconstructed tile and the matching half of the output; the partial scores
- * and the softmax weights P of Eq. mla_compact are exchanged between the two
- * through distributed shared memory, so every MMA spans all 128 query rows
- * (App. C.5 "cache update and tile reuse"; the split results are merged with
- * the "global attention normalization" rule as in qmla_mla_decode).
- * q_tokens x heads must be a multiple of 128 (QMLA_ERR_UNSUPPORTED otherwise);
- * layouts, workspace size (qmla_decode_workspace_bytes(batch, q_tokens *
- * heads)), results and errors as qmla_mla_decode_multi with prot_dev = NULL.
- * A wait of this kernel that runs out (2 s) sets QMLA_DEVERR_TIMEOUT and one
- * site bit among bits 17..27, and both CTAs of the pair leave. */
-int qmla_mla_decode_pair(const void* pool_dev, int c_bits, int num_blocks, const uint16_t* q_latent_dev,
-                         const uint16_t* q_pe_dev, int batch, int q_tokens, int heads,
-                         const int32_t* block_table_dev, int max_blocks, const int32_t* seq_lens_dev,
-                         float softmax_scale, float* out_dev, float* lse_dev, void* workspace_dev,
-                         size_t workspace_bytes, uint32_t* dev_err_dev, qmla_stream_t stream);
-
 /* The same decode over the BF16 comparison cache (same kernel, no dequantisation;
  * the paper's BF16 baseline, App. F.1). */
 int qmla_mla_decode_bf16cache(const void* pool_dev, int num_blocks, const uint16_t* q_latent_dev,
@@ -302,12 +284,55 @@ int qmla_mla_decode_c4r4(const void* pool_dev, int num_blocks, const uint16_t* q
                          float* out_dev, float* lse_dev, void* workspace_dev, size_t workspace_bytes,
                          uint32_t* dev_err_dev, qmla_stream_t stream);
 
-/* Measurement hook. While set (per host thread), every qmla_mla_decode* call
- * records the caller-owned CUDA events `before_main` and `after_main`
- * (cudaEvent_t, may be NULL) on its stream immediately before and after the
- * main decode kernel, so the caller can time that kernel alone with
- * cudaEventElapsedTime. Pass NULL, NULL to stop. Always returns QMLA_OK. */
-int qmla_set_profile_events(void* before_main, void* after_main);
+/*
+ * Every decode variant above from one descriptor (Eq. mla_compact; App. C.5):
+ * qmla_mla_decode, _protected, _c4r4, _multi and _bf16cache are this call with
+ * some fields fixed. Fields:
+ *   cache_kind      4 or 2 (this library's block at that content width),
+ *                   QMLA_CACHE_C4R4 (the paper's page) or QMLA_CACHE_BF16
+ *   pool, num_blocks, q_latent, q_pe, block_table, max_blocks, seq_lens,
+ *   softmax_scale, out, lse, workspace, workspace_bytes, dev_err
+ *                   as in qmla_mla_decode (q_latent / q_pe / out / lse shaped
+ *                   [batch, q_tokens, heads, ...] when q_tokens > 1)
+ *   batch, q_tokens, heads
+ *                   q_tokens 1..QMLA_MAX_Q_TOKENS query tokens per sequence,
+ *                   heads 1..128 per token (as qmla_mla_decode_multi)
+ *   prot            sink4/local128 protection buffer or NULL (not with BF16)
+ *   ev_before_main, ev_after_main
+ *                   optional cudaEvent_t (NULL = none): recorded on `stream`
+ *                   immediately before and after the main decode kernel of
+ *                   this call only, so that a caller can time that kernel
+ *                   with cudaEventElapsedTime. With either set, the call's
+ *                   launches wait for one another in full instead of
+ *                   overlapping their start-up, so that the events bracket
+ *                   the main kernel alone. The library keeps no reference to
+ *                   them after the call returns.
+ * Returns QMLA_ERR_INVALID_ARG for a NULL descriptor or a bad field, else as
+ * qmla_mla_decode. The descriptor is read during the call only.
+ */
+typedef struct qmla_decode_desc {
+  const void* pool;
+  int cache_kind;
+  int num_blocks;
+  const uint16_t* q_latent;
+  const uint16_t* q_pe;
+  int batch;
+  int q_tokens;
+  int heads;
+  const int32_t* block_table;
+  int max_blocks;
+  const int32_t* seq_lens;
+  const void* prot;
+  float softmax_scale;
+  float* out;
+  float* lse;
+  void* workspace;
+  size_t workspace_bytes;
+  uint32_t* dev_err;
+  void* ev_before_main;
+  void* ev_after_main;
+} qmla_decode_desc;
+int qmla_mla_decode_ex(const qmla_decode_desc* desc, qmla_stream_t stream);
 
 /* Bytes of the fixed device scratch array qmla_mla_decode_static uses
  * (32 MiB). */
@@ -328,13 +353,21 @@ size_t qmla_static_scratch_bytes(void);
  * - The first call on a device looks up that array's device address
  *   (cudaGetSymbolAddress) with the device current; make that first call
  *   before capturing any stream.
- * - Returns QMLA_ERR_WORKSPACE_TOO_SMALL when batch x heads need more scratch
- *   than the array holds (qmla_decode_workspace_bytes(batch, heads) >
- *   qmla_static_scratch_bytes(); e.g. up to 32 sequences at 128 heads).
+ * - Accepts batch x heads whose workspace fits the array:
+ *   qmla_decode_workspace_bytes(batch, heads) <= qmla_static_scratch_bytes().
+ *   Larger ones return QMLA_ERR_WORKSPACE_TOO_SMALL before any launch. The
+ *   workspace grows with the SM count; on a 152-SM GB300 32 sequences at 128
+ *   heads fit, 64 sequences at 128 heads do not.
  * - Every call shares the array, which keeps the last call's contents;
- *   nothing in it needs to start at zero (each call rewrites everything it
- *   reads). Calls whose work overlaps on the GPU (different streams, or
- *   different host threads on one device) race on it: serialise them.
+ *   nothing in it needs to start at zero (each call rewrites or clears
+ *   everything it reads). Calls whose work overlaps on the GPU (different
+ *   streams, or different host threads on one device) race on it: serialise
+ *   them.
+ * - The looked-up address is kept for the life of the process: after a
+ *   cudaDeviceReset of a device this entry point has run on, the address is
+ *   stale, so do not call it on that device again in the same process.
+ * - It is qmla_mla_decode_ex with the array as the workspace: argument checks
+ *   and errors are those of qmla_mla_decode.
  */
 int qmla_mla_decode_static(const void* pool_dev, int c_bits, int num_blocks, const uint16_t* q_latent_dev,
                            const uint16_t* q_pe_dev, int batch, int heads, const int32_t* block_table_dev,

@@ -25,6 +25,20 @@ DEVERR_BAD_SEQ = 4
 DEVERR_TIMEOUT = 8
 
 
+CACHE_KINDS = {4: 4, 2: 2, "c4r4": 5, "bf16": 16}  # qmla_decode_desc.cache_kind codes
+
+
+class DecodeDesc(ctypes.Structure):
+    """qmla_decode_desc (include/qmla.h), field for field."""
+    _fields_ = [("pool", ctypes.c_void_p), ("cache_kind", ctypes.c_int), ("num_blocks", ctypes.c_int),
+                ("q_latent", ctypes.c_void_p), ("q_pe", ctypes.c_void_p), ("batch", ctypes.c_int),
+                ("q_tokens", ctypes.c_int), ("heads", ctypes.c_int), ("block_table", ctypes.c_void_p),
+                ("max_blocks", ctypes.c_int), ("seq_lens", ctypes.c_void_p), ("prot", ctypes.c_void_p),
+                ("softmax_scale", ctypes.c_float), ("out", ctypes.c_void_p), ("lse", ctypes.c_void_p),
+                ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t), ("dev_err", ctypes.c_void_p),
+                ("ev_before_main", ctypes.c_void_p), ("ev_after_main", ctypes.c_void_p)]
+
+
 class QmlaError(RuntimeError):
     def __init__(self, fn: str, status: int):
         extra = ""
@@ -63,7 +77,7 @@ def lib():
     L.qmla_last_cuda_error.argtypes, L.qmla_last_cuda_error.restype = [], i32
     L.qmla_status_string.argtypes, L.qmla_status_string.restype = [i32], ctypes.c_char_p
     L.qmla_num_sms.argtypes, L.qmla_num_sms.restype = [], i32
-    L.qmla_set_profile_events.argtypes, L.qmla_set_profile_events.restype = [vp, vp], i32
+    L.qmla_mla_decode_ex.argtypes, L.qmla_mla_decode_ex.restype = [ctypes.POINTER(DecodeDesc), vp], i32
     L.qmla_static_scratch_bytes.argtypes, L.qmla_static_scratch_bytes.restype = [], sz
     L.qmla_mla_decode_static.argtypes = [vp, i32, i32, vp, vp, i32, i32, vp, i32, vp, f32, vp, vp, vp, vp]
     L.qmla_mla_decode_static.restype = i32
@@ -76,9 +90,6 @@ def lib():
     L.qmla_mla_decode_multi.argtypes = [vp, i32, i32, vp, vp, i32, i32, i32, vp, i32, vp, vp, f32, vp, vp, vp, sz,
                                         vp, vp]
     L.qmla_mla_decode_multi.restype = i32
-    L.qmla_mla_decode_pair.argtypes = [vp, i32, i32, vp, vp, i32, i32, i32, vp, i32, vp, f32, vp, vp, vp, sz, vp,
-                                       vp]
-    L.qmla_mla_decode_pair.restype = i32
     L.qmla_debug_wait_timeout.argtypes = [ctypes.c_uint32, vp, vp]
     L.qmla_debug_wait_timeout.restype = i32
     L.qmla_debug_tile.argtypes = [vp, i32, i32, vp, i32, vp, i32, i32, i32, vp, vp, vp, vp]
@@ -205,22 +216,6 @@ def mla_decode_multi(pool: torch.Tensor, c_bits: int, q_latent: torch.Tensor, q_
     _check("qmla_mla_decode_multi", st)
 
 
-def mla_decode_pair(pool: torch.Tensor, c_bits: int, q_latent: torch.Tensor, q_pe: torch.Tensor,
-                    block_table: torch.Tensor, seq_lens: torch.Tensor, softmax_scale: float, out: torch.Tensor,
-                    lse: torch.Tensor | None, workspace: torch.Tensor, dev_err: torch.Tensor, stream=None) -> None:
-    """qmla_mla_decode_pair: the decode on CTA pairs for q_tokens x heads a multiple of 128.
-    q_latent bf16 [B,H,512] or [B,T,H,512] (out, lse likewise); workspace for B x (T*H) heads."""
-    if q_latent.dim() == 3:
-        B, T, H = q_latent.shape[0], 1, q_latent.shape[1]
-    else:
-        B, T, H = q_latent.shape[0], q_latent.shape[1], q_latent.shape[2]
-    st = lib().qmla_mla_decode_pair(_ptr(pool), c_bits, pool.shape[0], _ptr(q_latent), _ptr(q_pe), B, T, H,
-                                    _ptr(block_table), block_table.shape[1], _ptr(seq_lens), float(softmax_scale),
-                                    _ptr(out), _ptr(lse), _ptr(workspace),
-                                    workspace.numel() * workspace.element_size(), _ptr(dev_err), _stream(stream))
-    _check("qmla_mla_decode_pair", st)
-
-
 CACHE_C4R4 = 5   # qmla_debug_tile cache kinds (besides content bit widths 4 and 2)
 CACHE_BF16 = 16
 
@@ -304,12 +299,28 @@ def static_scratch_bytes() -> int:
     return int(lib().qmla_static_scratch_bytes())
 
 
-def set_profile_events(before_main: torch.cuda.Event | None, after_main: torch.cuda.Event | None) -> None:
-    """qmla_set_profile_events: record these (already recorded once, so that
-    they exist) events around the main decode kernel of later decode calls."""
-    h0 = ctypes.c_void_p(before_main.cuda_event) if before_main is not None else None
-    h1 = ctypes.c_void_p(after_main.cuda_event) if after_main is not None else None
-    lib().qmla_set_profile_events(h0, h1)
+def mla_decode_ex(pool: torch.Tensor, cache_kind, q_latent: torch.Tensor, q_pe: torch.Tensor,
+                  block_table: torch.Tensor, seq_lens: torch.Tensor, softmax_scale: float, out: torch.Tensor,
+                  lse: torch.Tensor | None, workspace: torch.Tensor, dev_err: torch.Tensor, prot=None,
+                  events: tuple | None = None, stream=None) -> None:
+    """qmla_mla_decode_ex: cache_kind 4, 2, "c4r4" or "bf16"; q_latent [B,H,512] or
+    [B,T,H,512]; events = (before_main, after_main) torch.cuda.Event pair (already
+    recorded once, so that they exist) to record around this call's main kernel."""
+    if q_latent.dim() == 3:
+        B, T, H = q_latent.shape[0], 1, q_latent.shape[1]
+    else:
+        B, T, H = q_latent.shape[0], q_latent.shape[1], q_latent.shape[2]
+    d = DecodeDesc()
+    d.pool, d.cache_kind, d.num_blocks = _ptr(pool), CACHE_KINDS[cache_kind], pool.shape[0]
+    d.q_latent, d.q_pe, d.batch, d.q_tokens, d.heads = _ptr(q_latent), _ptr(q_pe), B, T, H
+    d.block_table, d.max_blocks, d.seq_lens = _ptr(block_table), block_table.shape[1], _ptr(seq_lens)
+    d.prot, d.softmax_scale, d.out, d.lse = _ptr(prot), float(softmax_scale), _ptr(out), _ptr(lse)
+    d.workspace, d.workspace_bytes = _ptr(workspace), workspace.numel() * workspace.element_size()
+    d.dev_err = _ptr(dev_err)
+    if events is not None:
+        d.ev_before_main = ctypes.c_void_p(events[0].cuda_event) if events[0] is not None else None
+        d.ev_after_main = ctypes.c_void_p(events[1].cuda_event) if events[1] is not None else None
+    _check("qmla_mla_decode_ex", lib().qmla_mla_decode_ex(ctypes.byref(d), _stream(stream)))
 
 
 def read_dev_err(dev_err: torch.Tensor, stream=None) -> int:

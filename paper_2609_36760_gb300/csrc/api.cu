@@ -11,8 +11,6 @@
 namespace {
 
 thread_local int g_last_cuda_error = 0;
-thread_local cudaEvent_t g_ev_before_main = nullptr;
-thread_local cudaEvent_t g_ev_after_main = nullptr;
 
 int cuda_fail(cudaError_t e) {
   g_last_cuda_error = static_cast<int>(e);
@@ -59,14 +57,14 @@ int append_common_checks(const void* pool, int num_blocks, const uint16_t* laten
   return QMLA_OK;
 }
 
-// heads counts every query row of a sequence (q_tokens x heads per token).
-int decode_common(const void* pool, int kind, int num_blocks, const uint16_t* q_latent, const uint16_t* q_pe,
-                  int batch, int heads, const int32_t* table, int max_blocks, const int32_t* seq_lens,
-                  float softmax_scale, float* out, float* lse, void* workspace, size_t workspace_bytes,
-                  uint32_t* dev_err, qmla_stream_t stream, const void* prot = nullptr, int q_tokens = 1,
-                  bool pair = false) {
+// Host checks of a decode call (no device access). heads counts every query
+// row of a sequence (q_tokens x heads per token).
+int decode_checks(const void* pool, int num_blocks, const uint16_t* q_latent, const uint16_t* q_pe, int batch,
+                  int heads, const int32_t* table, int max_blocks, const int32_t* seq_lens, float softmax_scale,
+                  const float* out, const float* lse, const void* workspace, const void* prot, int q_tokens,
+                  bool need_workspace = true) {
   if (pool == nullptr || q_latent == nullptr || q_pe == nullptr || table == nullptr || seq_lens == nullptr ||
-      out == nullptr || workspace == nullptr)
+      out == nullptr || (need_workspace && workspace == nullptr))
     return QMLA_ERR_INVALID_ARG;
   if (prot != nullptr && !aligned(prot, 16)) return QMLA_ERR_INVALID_ARG;
   if (q_tokens < 1 || q_tokens > QMLA_MAX_Q_TOKENS || heads % q_tokens != 0) return QMLA_ERR_INVALID_ARG;
@@ -75,11 +73,22 @@ int decode_common(const void* pool, int kind, int num_blocks, const uint16_t* q_
   if (!(softmax_scale > 0.0f) || softmax_scale > 1e30f) return QMLA_ERR_INVALID_ARG;
   if (!aligned(pool, 16) || !aligned(q_latent, 16) || !aligned(q_pe, 16) || !aligned(table, 4) ||
       !aligned(seq_lens, 4) || !aligned(out, 16) || (lse != nullptr && !aligned(lse, 4)) ||
-      !aligned(workspace, 256))
+      (need_workspace && !aligned(workspace, 256)))
     return QMLA_ERR_INVALID_ARG;
   if (static_cast<long long>(max_blocks) * qmla::kBlockTokens > INT32_MAX) return QMLA_ERR_INVALID_ARG;
+  return QMLA_OK;
+}
+
+int decode_common(const void* pool, int kind, int num_blocks, const uint16_t* q_latent, const uint16_t* q_pe,
+                  int batch, int heads, const int32_t* table, int max_blocks, const int32_t* seq_lens,
+                  float softmax_scale, float* out, float* lse, void* workspace, size_t workspace_bytes,
+                  uint32_t* dev_err, qmla_stream_t stream, const void* prot = nullptr, int q_tokens = 1,
+                  void* ev_before_main = nullptr, void* ev_after_main = nullptr) {
+  int st = decode_checks(pool, num_blocks, q_latent, q_pe, batch, heads, table, max_blocks, seq_lens, softmax_scale,
+                         out, lse, workspace, prot, q_tokens);
+  if (st != QMLA_OK) return st;
   DevInfo di;
-  int st = current_device_info(di);
+  st = current_device_info(di);
   if (st != QMLA_OK) return st;
   const qmla::DecodeWorkspace w = qmla::decode_workspace_layout(batch, heads, di.sms);
   if (workspace_bytes < w.total) return QMLA_ERR_WORKSPACE_TOO_SMALL;
@@ -102,17 +111,36 @@ int decode_common(const void* pool, int kind, int num_blocks, const uint16_t* q_
   a.grid = di.sms;
   a.prot = prot;
   a.q_tokens = q_tokens;
-  a.ev_before_main = g_ev_before_main;
-  a.ev_after_main = g_ev_after_main;
-  a.pair = pair;
+  a.ev_before_main = static_cast<cudaEvent_t>(ev_before_main);
+  a.ev_after_main = static_cast<cudaEvent_t>(ev_after_main);
   cudaError_t e = qmla::launch_decode(a, reinterpret_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
+}
+
+// Descriptor-level checks of qmla_mla_decode_ex before the common ones.
+int desc_checks(const qmla_decode_desc* d) {
+  if (d == nullptr) return QMLA_ERR_INVALID_ARG;
+  const int kind = d->cache_kind;
+  if (kind != 4 && kind != 2 && kind != QMLA_CACHE_C4R4 && kind != QMLA_CACHE_BF16) return QMLA_ERR_INVALID_ARG;
+  if (kind == QMLA_CACHE_BF16 && (d->prot != nullptr || d->q_tokens != 1)) return QMLA_ERR_INVALID_ARG;
+  if (kind == QMLA_CACHE_C4R4 && d->q_tokens != 1) return QMLA_ERR_INVALID_ARG;
+  if (d->q_tokens < 1 || d->q_tokens > QMLA_MAX_Q_TOKENS || d->heads < 1 || d->heads > 128)
+    return QMLA_ERR_INVALID_ARG;
+  return QMLA_OK;
 }
 
 }  // namespace
 
 namespace qmla {
 void record_cuda_error(int err) { g_last_cuda_error = err; }
+
+int check_decode_desc(const qmla_decode_desc* d, bool check_workspace) {
+  int st = desc_checks(d);
+  if (st != QMLA_OK) return st;
+  return decode_checks(d->pool, d->num_blocks, d->q_latent, d->q_pe, d->batch, d->q_tokens * d->heads,
+                       d->block_table, d->max_blocks, d->seq_lens, d->softmax_scale, d->out, d->lse, d->workspace,
+                       d->prot, d->q_tokens, check_workspace);
+}
 }  // namespace qmla
 
 extern "C" {
@@ -255,19 +283,6 @@ int qmla_mla_decode_multi(const void* pool_dev, int c_bits, int num_blocks, cons
                        workspace_bytes, dev_err_dev, stream, prot_dev, q_tokens);
 }
 
-int qmla_mla_decode_pair(const void* pool_dev, int c_bits, int num_blocks, const uint16_t* q_latent_dev,
-                         const uint16_t* q_pe_dev, int batch, int q_tokens, int heads,
-                         const int32_t* block_table_dev, int max_blocks, const int32_t* seq_lens_dev,
-                         float softmax_scale, float* out_dev, float* lse_dev, void* workspace_dev,
-                         size_t workspace_bytes, uint32_t* dev_err_dev, qmla_stream_t stream) {
-  if (c_bits != 4 && c_bits != 2) return QMLA_ERR_INVALID_ARG;
-  if (q_tokens < 1 || q_tokens > QMLA_MAX_Q_TOKENS || heads < 1 || heads > 128) return QMLA_ERR_INVALID_ARG;
-  if ((q_tokens * heads) % 128 != 0) return QMLA_ERR_UNSUPPORTED;
-  return decode_common(pool_dev, c_bits, num_blocks, q_latent_dev, q_pe_dev, batch, q_tokens * heads,
-                       block_table_dev, max_blocks, seq_lens_dev, softmax_scale, out_dev, lse_dev, workspace_dev,
-                       workspace_bytes, dev_err_dev, stream, nullptr, q_tokens, true);
-}
-
 int qmla_mla_decode_bf16cache(const void* pool_dev, int num_blocks, const uint16_t* q_latent_dev,
                               const uint16_t* q_pe_dev, int batch, int heads, const int32_t* block_table_dev,
                               int max_blocks, const int32_t* seq_lens_dev, float softmax_scale, float* out_dev,
@@ -327,10 +342,13 @@ int qmla_read_dev_err(const uint32_t* dev_err_dev, uint32_t* host_out, qmla_stre
   return e == cudaSuccess ? QMLA_OK : cuda_fail(e);
 }
 
-int qmla_set_profile_events(void* before_main, void* after_main) {
-  g_ev_before_main = static_cast<cudaEvent_t>(before_main);
-  g_ev_after_main = static_cast<cudaEvent_t>(after_main);
-  return QMLA_OK;
+int qmla_mla_decode_ex(const qmla_decode_desc* d, qmla_stream_t stream) {
+  const int st = desc_checks(d);
+  if (st != QMLA_OK) return st;
+  return decode_common(d->pool, d->cache_kind, d->num_blocks, d->q_latent, d->q_pe, d->batch, d->q_tokens * d->heads,
+                       d->block_table, d->max_blocks, d->seq_lens, d->softmax_scale, d->out, d->lse, d->workspace,
+                       d->workspace_bytes, d->dev_err, stream, d->prot, d->q_tokens, d->ev_before_main,
+                       d->ev_after_main);
 }
 
 int qmla_last_cuda_error(void) { return g_last_cuda_error; }

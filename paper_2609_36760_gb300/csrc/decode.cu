@@ -142,8 +142,6 @@ template <int HG>
 struct Cfg {
   static constexpr int kQBytes = kNumChunks * HG * 128;
   // O^T (4 HG columns) and S^T (HG), rounded up to a power of 2.
-  // (HG = 128 is the unit of the cluster-pair kernel, which has its own
-  // layout; only the prep and merge kernels are instantiated for it.)
   static constexpr uint32_t kTmemCols = HG >= 64 ? 512 : (HG == 32 ? 256 : 128);
   static_assert(HG > 64 || 5 * HG <= static_cast<int>(kTmemCols), "TMEM columns");
   static constexpr int kSmem = 1024 + kNumChunks * kChunkBytes + kQBytes + (int)sizeof(Ctrl);
@@ -1624,7 +1622,6 @@ cudaError_t launch_k(void (*kern)(Args...), dim3 grid, dim3 block, size_t smem, 
   return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
-#include "decode_pair.cuh"
 
 template <int CB, int HG, bool PROT>
 cudaError_t launch_impl(const Params& prm, cudaStream_t stream, cudaEvent_t ev0, cudaEvent_t ev1) {
@@ -1727,10 +1724,6 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream) {
   prm.trace = nullptr;
 #endif
   const bool prot = prm.prot != nullptr;
-  if (a.pair) {  // units of 128 query rows on CTA pairs (INT4 / INT2 block, no protection)
-    return a.cache_kind == 2 ? launch_pair_impl<2>(prm, a.grid, stream, a.ev_before_main, a.ev_after_main)
-                             : launch_pair_impl<4>(prm, a.grid, stream, a.ev_before_main, a.ev_after_main);
-  }
   if (a.cache_kind == kC4R4)
     return prot ? launch_hg<kC4R4, true>(hg, prm, stream, a.ev_before_main, a.ev_after_main)
                 : launch_hg<kC4R4, false>(hg, prm, stream, a.ev_before_main, a.ev_after_main);

@@ -4,6 +4,8 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
+#include "qmla.h"
+
 namespace qmla {
 
 // c_bits: 4 or 2 (this library's block) or kC4R4 (the paper's page).
@@ -47,9 +49,6 @@ struct DecodeArgs {
   const void* prot = nullptr;  // sink4/local128 protection buffer, or null
   cudaEvent_t ev_before_main = nullptr;  // optional, recorded around the main kernel
   cudaEvent_t ev_after_main = nullptr;
-  // Cluster-pair kernel: units of 128 query rows (heads a multiple of 128),
-  // cache_kind 4 or 2, no protection buffer.
-  bool pair = false;
 };
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t stream);
 // Test hook: tile j of sequence b as the decode kernel builds it, [128][576] fp16.
@@ -59,6 +58,9 @@ cudaError_t launch_wait_timeout(uint32_t* dev_err, unsigned long long limit_ns, 
 
 // Records a failed CUDA call for qmla_last_cuda_error (calling thread).
 void record_cuda_error(int err);
+// The host checks of qmla_mla_decode_ex (no device access); the workspace
+// fields are checked only with check_workspace.
+int check_decode_desc(const qmla_decode_desc* d, bool check_workspace);
 
 #ifdef QMLA_TRACE_BUILD
 // Trace builds only: device buffer of [8 CTAs][96 events][32 tiles] u64 clock64 stamps.

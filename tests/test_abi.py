@@ -107,21 +107,45 @@ def test_multi_query_host_checks(libqmla):
     assert L.qmla_mla_decode_multi(*args) == 1
 
 
-def test_pair_decode_host_checks(libqmla):
+def _desc(**kw):
+    import paper_2609_36760_gb300 as Q
+    fake = 0x10000
+    d = Q.DecodeDesc()
+    d.pool, d.cache_kind, d.num_blocks = fake, 4, 4
+    d.q_latent, d.q_pe, d.batch, d.q_tokens, d.heads = fake, fake, 1, 1, 16
+    d.block_table, d.max_blocks, d.seq_lens = fake, 1, fake
+    d.prot, d.softmax_scale, d.out, d.lse = None, 0.1, fake, None
+    d.workspace, d.workspace_bytes, d.dev_err = fake, 1 << 30, None
+    for k, v in kw.items():
+        setattr(d, k, v)
+    return d
+
+
+def test_decode_ex_host_checks(libqmla):
+    L = libqmla
+    assert L.qmla_mla_decode_ex(None, None) == 1                       # no descriptor
+    for bad in ({"cache_kind": 3}, {"cache_kind": 8}, {"q_tokens": 0}, {"q_tokens": 9}, {"heads": 0},
+                {"heads": 129}, {"batch": 0}, {"out": None}, {"workspace": None}, {"softmax_scale": -1.0},
+                {"pool": 0x10008}, {"workspace": 0x10010}, {"prot": 0x10008},
+                {"cache_kind": 16, "prot": 0x10000},                     # no protection on the BF16 cache
+                {"cache_kind": 16, "q_tokens": 2}, {"cache_kind": 5, "q_tokens": 2}):
+        d = _desc(**bad)
+        assert L.qmla_mla_decode_ex(ctypes.byref(d), None) == 1, bad
+
+
+def test_static_decode_host_checks(libqmla):
+    # The allocation-free entry point rejects bad arguments before any device
+    # call (so these run without a GPU): bits, heads, batch, pointers, scale,
+    # alignment, table size.
     L = libqmla
     fake = ctypes.c_void_p(0x10000)
-    base = [fake, 4, 4, fake, fake, 1, 1, 128, fake, 1, fake, 0.1, fake, None, fake, 1 << 30, None, None]
-    for i, bad in ((1, 3), (6, 0), (6, 9), (7, 0), (7, 129)):   # c_bits, q_tokens, heads
+    base = [fake, 4, 4, fake, fake, 1, 16, fake, 1, fake, 0.1, fake, None, None, None]
+    for i, bad in ((1, 3), (1, 8), (6, 0), (6, 129), (5, 0), (0, None), (3, None), (7, None), (9, None),
+                   (11, None), (10, -1.0), (10, 0.0), (0, ctypes.c_void_p(0x10008)),
+                   (3, ctypes.c_void_p(0x10004)), (11, ctypes.c_void_p(0x10004)), (8, 1 << 26)):
         args = list(base)
         args[i] = bad
-        assert L.qmla_mla_decode_pair(*args) == 1, (i, bad)
-    for T, H in ((1, 64), (3, 100), (1, 16)):                     # T x H not a multiple of 128
-        args = list(base)
-        args[6], args[7] = T, H
-        assert L.qmla_mla_decode_pair(*args) == 2, (T, H)
-    args = list(base)
-    args[12] = None                                               # no output
-    assert L.qmla_mla_decode_pair(*args) == 1
+        assert L.qmla_mla_decode_static(*args) == 1, (i, bad)
 
 
 def test_debug_hooks_host_checks(libqmla):

@@ -206,3 +206,79 @@ def test_serving_mix_256_steps():
             out, lse = c.decode(step)
             check(c, step, seqs, out, lse)
     assert c.dev_error() == 0
+
+
+def test_many_units_split_over_many_pieces():
+    # 40 units of ragged length: one long sequence spans dozens of CTAs, most
+    # units are split over several; empty, one-token and too-long sequences sit
+    # between split ones.
+    rng = np.random.default_rng(7)
+    lengths = [int(x) for x in rng.integers(100, 3000, size=40)]
+    lengths[3], lengths[11], lengths[20], lengths[33] = 30000, 0, 1, 0
+    w = W.small_workload("fuse", batch=40, heads=64, lengths=lengths, seed=93)
+    c = Case(w)
+    c.prefill_all()
+    lens = list(lengths)
+    lens[35] = 64 * (c.table_d.shape[1] + 3)  # beyond its table: an error bit, then out 0 / lse -inf
+    out, lse = c.decode(0, lens=lens)
+    assert c.dev_error() & Q.DEVERR_BAD_POSITION
+    for b in (11, 33, 35):
+        assert np.all(out[b] == 0) and np.all(np.isneginf(lse[b]))
+    check_tile(c, 0, [20], out, lse)
+    seqs = [0, 3, 7, 19, 21, 39]
+    lens_ok = c.lengths_at(0)
+    outs, refs = [], []
+    for b in seqs:
+        ref, rlse = c.oracle_decode(b, lens_ok[b], 0)
+        outs.append(out[b]); refs.append(ref)
+        assert np.max(np.abs(lse[b] - rlse)) <= LSE_ABS
+    o, r = np.stack(outs), np.stack(refs)
+    assert np.max(np.abs(o - r)) <= MAX_ABS and rel_l2(o, r) <= REL_L2
+
+
+def test_decode_ex_matches_entry_points():
+    # qmla_mla_decode_ex with a descriptor is the same computation as the
+    # per-variant entry points: identical bits for the INT4 block and the BF16 cache.
+    for bf16 in (False, True):
+        w = W.small_workload("ex", batch=5, heads=64, lengths=(1, 200, 4097, 900, 64), seed=95)
+        c = Case(w, bf16_cache=bf16)
+        c.prefill_all()
+        ref_out, ref_lse = c.decode(0)
+        ql, qp = W.queries(w, 0)
+        out = torch.full((w.batch, w.heads, 512), float("nan"), dtype=torch.float32, device="cuda")
+        lse = torch.full((w.batch, w.heads), float("nan"), dtype=torch.float32, device="cuda")
+        ws = Q.workspace_for(w.batch, w.heads, "cuda")
+        sl = torch.tensor(c.lengths_at(0), dtype=torch.int32, device="cuda")
+        Q.mla_decode_ex(c.pool, "bf16" if bf16 else 4, ql.cuda(), qp.cuda(), c.table_d, sl, TAU, out, lse, ws,
+                        c.dev_err)
+        torch.cuda.synchronize()
+        assert np.array_equal(out.cpu().numpy(), ref_out) and np.array_equal(lse.cpu().numpy(), ref_lse)
+        assert c.dev_error() == 0
+
+
+def test_decode_ex_events_are_per_call():
+    # Events given to one call bracket that call's main kernel only: a call in
+    # between without events leaves them alone (no state survives the call).
+    w = W.small_workload("evt", batch=8, heads=128, lengths=(4000,), seed=97)
+    c = Case(w)
+    c.prefill_all()
+    ql, qp = W.queries(w, 0)
+    ql, qp = ql.cuda(), qp.cuda()
+    out = torch.empty((w.batch, w.heads, 512), dtype=torch.float32, device="cuda")
+    lse = torch.empty((w.batch, w.heads), dtype=torch.float32, device="cuda")
+    ws = Q.workspace_for(w.batch, w.heads, "cuda")
+    sl = torch.tensor(c.lengths_at(0), dtype=torch.int32, device="cuda")
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    for e in ev:
+        e.record()
+    torch.cuda.synchronize()
+    Q.mla_decode_ex(c.pool, 4, ql, qp, c.table_d, sl, TAU, out, lse, ws, c.dev_err, events=(ev[0], ev[1]))
+    Q.mla_decode(c.pool, 4, ql, qp, c.table_d, sl, TAU, out, lse, ws, c.dev_err)
+    Q.mla_decode_ex(c.pool, 4, ql, qp, c.table_d, sl, TAU, out, lse, ws, c.dev_err, events=(ev[2], ev[3]))
+    torch.cuda.synchronize()
+    first, second = ev[0].elapsed_time(ev[1]), ev[2].elapsed_time(ev[3])
+    between = ev[1].elapsed_time(ev[2])
+    assert first > 0 and second > 0
+    # the middle call's main kernel runs between the two brackets
+    assert between > 0.5 * min(first, second), (first, between, second)
+    assert c.dev_error() == 0

@@ -63,8 +63,12 @@ class Workload:
         return self.heads
 
 
-def _gen(seed: int, stream: int) -> torch.Generator:
-    g = torch.Generator(device="cpu")
+def _gen(seed: int, stream: int, device=None) -> torch.Generator:
+    """The seeded generator of one stream. On the CPU (the default) it gives the
+    values every test and the oracle use; on a CUDA device the same recipe gives
+    other values from the same distributions (bench.py's secondary workloads,
+    whose inputs are too large to draw quickly on the host)."""
+    g = torch.Generator(device="cpu" if device is None else device)
     g.manual_seed(seed * 10_000_019 + stream)
     return g
 
@@ -97,44 +101,47 @@ def channel_gains(w: Workload) -> torch.Tensor:
     return gain
 
 
-def latent_for_seq(w: Workload, b: int, n_tokens: int, gains: torch.Tensor | None = None) -> torch.Tensor:
-    """Content latent rows 0..n_tokens-1 of sequence ``b`` as bf16 [n, 512]."""
-    g = _gen(w.seed, _S_LATENT_BASE + b)
+def latent_for_seq(w: Workload, b: int, n_tokens: int, gains: torch.Tensor | None = None,
+                   device=None) -> torch.Tensor:
+    """Content latent rows 0..n_tokens-1 of sequence ``b`` as bf16 [n, 512]
+    (drawn on ``device``, see _gen)."""
+    g = _gen(w.seed, _S_LATENT_BASE + b, device)
     if gains is None:
         gains = channel_gains(w)
+    gains = gains.to(g.device)
     if w.latent_dist == "gauss_gain_outlier":
-        x = torch.randn(n_tokens, D_C, generator=g, dtype=torch.float64)
+        x = torch.randn(n_tokens, D_C, generator=g, dtype=torch.float64, device=g.device)
     else:  # Student-t with 4 degrees of freedom: N / sqrt(chi2_4 / 4),
         # chi2_4 = -2 ln(U1 U2) (a sum of two exponentials with mean 2)
-        z = torch.randn(n_tokens, D_C, generator=g, dtype=torch.float64)
-        u = 1.0 - torch.rand(2, n_tokens, D_C, generator=g, dtype=torch.float64)
+        z = torch.randn(n_tokens, D_C, generator=g, dtype=torch.float64, device=g.device)
+        u = 1.0 - torch.rand(2, n_tokens, D_C, generator=g, dtype=torch.float64, device=g.device)
         chi = -2.0 * (torch.log(u[0]) + torch.log(u[1]))
         x = z / torch.sqrt(chi / 4.0)
     return (x * gains).to(torch.bfloat16)
 
 
-def kpe_for_seq(w: Workload, b: int, n_tokens: int, theta: float = 10000.0) -> torch.Tensor:
+def kpe_for_seq(w: Workload, b: int, n_tokens: int, theta: float = 10000.0, device=None) -> torch.Tensor:
     """RoPE key rows 0..n_tokens-1 of sequence ``b`` as bf16 [n, 64].
 
     Token i sits at position i; the pair (j, j + 32) is rotated by the angle
     i * theta^(-2j/64).
     """
-    g = _gen(w.seed, _S_KPE_BASE + b)
-    x = torch.randn(n_tokens, D_R, generator=g, dtype=torch.float64)
+    g = _gen(w.seed, _S_KPE_BASE + b, device)
+    x = torch.randn(n_tokens, D_R, generator=g, dtype=torch.float64, device=g.device)
     half = D_R // 2
-    inv_freq = theta ** (-2.0 * torch.arange(half, dtype=torch.float64) / D_R)
-    ang = torch.arange(n_tokens, dtype=torch.float64)[:, None] * inv_freq[None, :]
+    inv_freq = theta ** (-2.0 * torch.arange(half, dtype=torch.float64, device=g.device) / D_R)
+    ang = torch.arange(n_tokens, dtype=torch.float64, device=g.device)[:, None] * inv_freq[None, :]
     cos, sin = torch.cos(ang), torch.sin(ang)
     x1, x2 = x[:, :half], x[:, half:]
     out = torch.cat([x1 * cos - x2 * sin, x1 * sin + x2 * cos], dim=1)
     return out.to(torch.bfloat16)
 
 
-def queries(w: Workload, step: int = 0) -> tuple[torch.Tensor, torch.Tensor]:
+def queries(w: Workload, step: int = 0, device=None) -> tuple[torch.Tensor, torch.Tensor]:
     """(q_latent [B,H,512], q_pe [B,H,64]) as bf16 for decode step ``step``."""
-    g = _gen(w.seed, _S_QUERY + 7919 * step)
-    ql = torch.randn(w.batch, w.heads, D_C, generator=g, dtype=torch.float64) / math.sqrt(D_C)
-    qp = torch.randn(w.batch, w.heads, D_R, generator=g, dtype=torch.float64) / math.sqrt(D_R)
+    g = _gen(w.seed, _S_QUERY + 7919 * step, device)
+    ql = torch.randn(w.batch, w.heads, D_C, generator=g, dtype=torch.float64, device=g.device) / math.sqrt(D_C)
+    qp = torch.randn(w.batch, w.heads, D_R, generator=g, dtype=torch.float64, device=g.device) / math.sqrt(D_R)
     return ql.to(torch.bfloat16), qp.to(torch.bfloat16)
 
 
