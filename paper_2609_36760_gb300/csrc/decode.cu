@@ -588,6 +588,33 @@ __device__ __forceinline__ void store_row_bf16(uint32_t chunk_base, int row, con
   }
 }
 
+// BF16 cache rows read coalesced: lane l of a warp handles piece l & 7 (16
+// bytes) of rows r0 + 4 i + (l >> 3), i = 0..7, so every load instruction
+// reads four whole 128-byte lines (32 rows x one chunk per warp). r0 is the
+// warp's first row (its rows share a block, slots slot0 ..); vmask bit m is
+// set when row r0 + m is to be read (else zeros).
+__device__ __forceinline__ void bf16_load_t(uint4 (&v)[8], const uint8_t* blk, uint32_t vmask, int slot0, int k,
+                                            int lane) {
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int m = 4 * i + (lane >> 3);
+    v[i] = (vmask >> m) & 1u ? ldg_nc_v4(blk + (slot0 + m) * (kDqk * 2) + k * 128 + (lane & 7) * 16)
+                             : make_uint4(0, 0, 0, 0);
+  }
+}
+// Writes those pieces rounded to fp16 into the swizzled chunk.
+__device__ __forceinline__ void bf16_store_t(uint32_t chunk_base, int r0, const uint4 (&v)[8], int lane) {
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int m = 4 * i + (lane >> 3);
+    const uint32_t w[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+    uint32_t o[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) o[e] = pack_h2(bf16_lo(w[e]), bf16_hi(w[e]));
+    sts_v4(chunk_base + swz_off(r0 + m, lane & 7, 128), o[0], o[1], o[2], o[3]);
+  }
+}
+
 // Query image of one unit: HG heads x 576 channels in fp16 laid out exactly as
 // the K-major, 128-byte-swizzled shared-memory operand ([chunk][head][128 B]),
 // channels permuted within each 8-channel piece like the cache rows. Piece
@@ -904,9 +931,10 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       if (k < kNumChunks) f[kc] = fetch_chunk<CB>(blk_cur, valid_cur, k, slot);
     }
   } else {
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-      cur[i] = valid_cur ? ldg_nc_v4(blk_cur + slot * (kDqk * 2) + par * 128 + i * 16) : make_uint4(0, 0, 0, 0);
+    // (the warp's 32 rows share a block: lane 0's row is valid whenever any is)
+    const uint8_t* wblk = reinterpret_cast<const uint8_t*>(
+        __shfl_sync(0xffffffffu, reinterpret_cast<unsigned long long>(blk_cur), 0));
+    bf16_load_t(cur, wblk, __ballot_sync(0xffffffffu, valid_cur), slot & ~31, par, lane);
   }
   // Table references run one tile ahead of the block pointer they resolve to.
   Sched nx = sc;
@@ -929,6 +957,18 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       }
     }
     const uint8_t* blk_nx = psrc_nx != nullptr ? nullptr : resolve_row<CB>(p, ref_nx, row, valid_nx);
+    if constexpr (CB == 16) {
+      // BF16 cache: its rows are read only one chunk ahead into registers, so
+      // bring the next tile's lines of this thread's row and chunks into L2 now.
+      if (valid_nx) {
+#pragma unroll
+        for (int kc = 0; kc < kMyChunks; ++kc) {
+          const int k = 2 * kc + par;
+          if (k < kNumChunks)
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(blk_nx + slot * (kDqk * 2) + k * 128));
+        }
+      }
+    }
     Sched nn = nx;
     nn.next();
     const RowRef ref_nn = row_ref(p, nn, row);
@@ -950,16 +990,12 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       if constexpr (CB == 16) {
         uint4 nxt[8];
         const int kn = k + 2;
-        if (kn < kNumChunks) {
-#pragma unroll
-          for (int i = 0; i < 8; ++i)
-            nxt[i] = valid_cur ? ldg_nc_v4(blk_cur + slot * (kDqk * 2) + kn * 128 + i * 16) : make_uint4(0, 0, 0, 0);
-        } else {
-#pragma unroll
-          for (int i = 0; i < 8; ++i)
-            nxt[i] = valid_nx ? ldg_nc_v4(blk_nx + slot * (kDqk * 2) + par * 128 + i * 16) : make_uint4(0, 0, 0, 0);
-        }
-        store_row_bf16(chunks + k * kChunkBytes, row, cur, valid_cur);
+        const bool same = kn < kNumChunks;  // the next chunk of this tile, else the next tile's first
+        const uint8_t* wblk = reinterpret_cast<const uint8_t*>(__shfl_sync(
+            0xffffffffu, reinterpret_cast<unsigned long long>(same ? blk_cur : blk_nx), 0));
+        bf16_load_t(nxt, wblk, __ballot_sync(0xffffffffu, same ? valid_cur : valid_nx), slot & ~31,
+                    same ? kn : par, lane);
+        bf16_store_t(chunks + k * kChunkBytes, q4 * 32, cur, lane);
 #pragma unroll
         for (int i = 0; i < 8; ++i) cur[i] = nxt[i];
       } else {
