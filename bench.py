@@ -173,15 +173,20 @@ def profile_traffic(kernel_file_hash: str):
     return d
 
 
+# The sources decode_main is compiled from (its translation unit and headers).
+DECODE_MAIN_SOURCES = ("common.cuh", "decode.cu", "kernels.h", "ptx.cuh")
+
+
 def decode_cu_hash() -> str:
-    """sha256 over every CUDA source and header of the library (sorted by name),
-    so a traffic figure taken on another version of the kernel is not used."""
+    """sha256 over the sources decode_main is compiled from (and the public
+    header they include), so a traffic figure taken on another version of the
+    kernel is not used."""
     d = os.path.join(ROOT, "paper_2609_36760_gb300", "csrc")
     h = hashlib.sha256()
-    for name in sorted(os.listdir(d)):
-        if name.endswith((".cu", ".cuh", ".h")):
-            with open(os.path.join(d, name), "rb") as f:
-                h.update(name.encode() + b"\0" + f.read())
+    paths = [os.path.join(d, n) for n in DECODE_MAIN_SOURCES] + [os.path.join(ROOT, "include", "qmla.h")]
+    for path in paths:
+        with open(path, "rb") as f:
+            h.update(os.path.basename(path).encode() + b"\0" + f.read())
     return h.hexdigest()
 
 
@@ -712,8 +717,10 @@ def main_trace_summary(ev):
     """Median stage lengths (cycles) of decode_main's steady tiles (2 .. n-2 of
     each traced CTA). Event numbers as stamped in decode.cu: MMA thread 112 + k
     QK of chunk k issued, 12 QK committed, 14 P seen, 15 PV issued; worker warp
-    0: 0 loop top, 16 scores seen, 19 P written, 17 every warp's P seen;
-    lane 0 of warp w: 88 + w last slot wait passed, 32 + w tile dequantised."""
+    0: 0 loop top, 16 scores seen, 19 P written, 17 every warp's P seen, 18 row
+    sums added; lane 0 of warp w: 88 + w last slot wait passed, 32 + w tile
+    dequantised, 48 + 5 w + kc chunk step kc arrived; warp 0 (4) also 105 + kc
+    (-) chunk computed and 96 + kc (101 + kc) its slot wait passed."""
     import numpy as np
 
     stages, period = {}, []
@@ -732,8 +739,6 @@ def main_trace_summary(ev):
                             ("warp0: P written -> all P seen", g[17] - g[19]),
                             ("warp0: all P seen -> row sums added", g[18] - g[17]),
                             ("warp0: row sums added -> next loop top", nx[0] - g[18]),
-                            ("dequant: PV issued -> last slot wait passed (max warp)",
-                             max(nx[88 + w] for w in range(8)) - g[15]),
                             ("dequant: PV issued -> tile dequantised (max warp)",
                              max(nx[32 + w] for w in range(8)) - g[15])):
                 stages.setdefault(name, []).append(v)
