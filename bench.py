@@ -160,9 +160,11 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def profile_traffic(kernel_file_hash: str):
-    """DRAM bytes per main-kernel launch from the committed ncu summary, if it
-    was taken on the current kernel source; otherwise None."""
+def profile_traffic(kernel_file_hash: str, workload: str, bf16: bool = False, protect: bool = False,
+                    c4r4: bool = False, q_tokens: int = 1):
+    """The committed ncu record of DRAM bytes per main-kernel launch for this
+    workload and cache variant, if it was taken on the current kernel sources;
+    otherwise None."""
     p = os.path.join(ROOT, "profiles", "decode_main_traffic.json")
     if not os.path.exists(p):
         return None
@@ -170,7 +172,12 @@ def profile_traffic(kernel_file_hash: str):
         d = json.load(f)
     if d.get("decode_cu_sha256") != kernel_file_hash:
         return None
-    return d
+    for r in d.get("records", []):
+        if (r.get("workload") == workload and bool(r.get("bf16_cache")) == bool(bf16)
+                and bool(r.get("protect")) == bool(protect) and bool(r.get("c4r4")) == bool(c4r4)
+                and int(r.get("q_tokens", 1)) == q_tokens):
+            return r
+    return None
 
 
 # The sources decode_main is compiled from (its translation unit and headers).
@@ -424,14 +431,11 @@ def run_native(args, ws_world: int, rank: int, local: int):
     value = whole_job_value(ws_world, tok_per_step, ms_step_max)
 
     roof = roofline(w, t["lens0"], args.bf16_cache, state.c4r4, args.q_tokens, ms_main)
-    prof = profile_traffic(decode_cu_hash())
-    roof["traffic"] = (prof["dram_bytes_per_launch"] if prof and prof.get("workload") == args.workload
-                       and bool(prof.get("bf16_cache")) == bool(args.bf16_cache)
-                       and bool(prof.get("protect")) == bool(args.protect)
-                       and bool(prof.get("c4r4")) == bool(state.c4r4)
-                       and int(prof.get("q_tokens", 1)) == args.q_tokens else None)
-    if roof["traffic"] is not None:
-        roof["traffic_source"] = prof.get("source", "profiles/decode_main_traffic.json")
+    prof = profile_traffic(decode_cu_hash(), args.workload, args.bf16_cache, args.protect, state.c4r4,
+                           args.q_tokens)
+    roof["traffic"] = prof["dram_bytes_per_launch"] if prof else None
+    if prof:
+        roof["traffic_source"] = "profiles/decode_main_traffic.json: " + prof["source"]
     roof["kernel"] = "decode_main"
 
     # end to end through the public API with host buffers
@@ -502,6 +506,8 @@ def run_configs(dev, flush, K: int) -> dict:
         ms_step = sum(step_ms) / len(step_ms)
         ms_main = sum(main_ms) / len(main_ms)
         roof = roofline(state.w, t["lens0"], bf16, False, 1, ms_main)
+        prof = profile_traffic(decode_cu_hash(), name, bf16)
+        roof["traffic"] = prof["dram_bytes_per_launch"] if prof else None
         qs = statistics.quantiles(step_ms, n=10) if len(step_ms) >= 10 else [min(step_ms)] * 9
         r = {"cache": cache_name(w, bf16, False, False), "batch": w.batch, "heads": w.heads,
              "steps": Kc, "warmup": Wc, "us_per_step": round(ms_step * 1e3, 2),
@@ -510,7 +516,7 @@ def run_configs(dev, flush, K: int) -> dict:
              "kv_tokens_per_s": round(t["tokens_per_step"] / (ms_step * 1e-3), 1),
              "kv_tokens_per_step": t["tokens_per_step"], "step_parts_us": t["parts_us"],
              "roofline": {k: roof[k] for k in ("bound", "achieved", "peak", "unit", "frac", "kernel_us",
-                                              "roofline_us", "algorithmic_bytes", "algorithmic_flops")},
+                                              "roofline_us", "algorithmic_bytes", "algorithmic_flops", "traffic")},
              "hbm_gbs_of_step": round(roof["algorithmic_bytes"] / (ms_step * 1e-3) / 1e9, 1),
              "gpu_launches": state.launches_per_step() * Kc,
              "inputs": "seeded, drawn on the GPU (same distributions as workloads/synthetic.py)"}
