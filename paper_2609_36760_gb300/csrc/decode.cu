@@ -477,10 +477,6 @@ __device__ __forceinline__ void dq_regs(uint32_t (&o)[32], const Fetch& f, bool 
       o[4 * i + 3] = dq2(__byte_perm((x >> 6) & 0x03030303u, K, sel), zz, ss);
     }
   }
-  // Pin the results here: the (volatile) slot wait that follows must not be
-  // hoisted above the arithmetic.
-#pragma unroll
-  for (int i = 0; i < 32; ++i) asm volatile("" : "+r"(o[i]));
 }
 __device__ __forceinline__ void store_regs(uint32_t chunk_base, int row, const uint32_t (&o)[32]) {
 #pragma unroll
@@ -586,6 +582,43 @@ __device__ __forceinline__ void store_row_bf16(uint32_t chunk_base, int row, con
     }
     sts_v4(chunk_base + swz_off(row, i, 128), o[0], o[1], o[2], o[3]);
   }
+}
+
+// One row's chunk k of this library's block as dq_row would store it (the
+// eight 16-byte pieces in order), computed into registers: the protected bf16
+// row when ps is set, else the packed row f. The decode workers compute it
+// before waiting for the chunk's slot, so only the stores follow the slot's
+// release.
+template <int CB, bool PROT>
+__device__ __forceinline__ void row_regs(uint32_t (&o)[32], const Fetch& f, int k, const uint8_t* ps) {
+  if (PROT && ps != nullptr) {
+    uint4 pv[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) pv[i] = __ldg(reinterpret_cast<const uint4*>(ps + k * 128) + i);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t w[4] = {pv[i].x, pv[i].y, pv[i].z, pv[i].w};
+      float v[8];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        v[2 * e] = bf16_lo(w[e]);
+        v[2 * e + 1] = bf16_hi(w[e]);
+      }
+      if (k < 8) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) o[4 * i + e] = pack_h2(v[Perm<CB>::at(2 * e)], v[Perm<CB>::at(2 * e + 1)]);
+      } else {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) o[4 * i + e] = pack_h2(v[Perm<4>::at(2 * e)], v[Perm<4>::at(2 * e + 1)]);
+      }
+    }
+  } else {
+    dq_regs(o, f, CB == 4 || k == 8);
+  }
+  // Pin the results here: the (volatile) slot wait that follows must not be
+  // hoisted above the arithmetic.
+#pragma unroll
+  for (int i = 0; i < 32; ++i) asm volatile("" : "+r"(o[i]));
 }
 
 // BF16 cache rows read coalesced: lane l of a warp handles piece l & 7 (16
@@ -975,14 +1008,15 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     if (lane == 0 && warp == 0) QMLA_TRACE(0, it);
 
     // ---- dequantise this tile, chunk by chunk as the previous PV frees the slots
-    // (this library's INT4 / INT2 block: the arithmetic before the slot wait)
-    constexpr bool kEarly = (CB == 4 || CB == 2) && !PROT;
+    // (this library's INT4 / INT2 block, protected rows included: each row's
+    // chunk computed before its slot wait; measured no faster for the paper's page)
+    constexpr bool kEarly = CB == 4 || CB == 2;
 #pragma unroll
     for (int kc = 0; kc < kMyChunks; ++kc) {
       const int k = 2 * kc + par;
       if (k >= kNumChunks) break;
       uint32_t dq[kEarly ? 32 : 1];
-      if constexpr (kEarly) dq_regs(dq, f[kc], CB == 4 || k == 8);
+      if constexpr (kEarly) row_regs<CB, PROT>(dq, f[kc], k, psrc_cur);
       if (lane == 0 && warp == 0) QMLA_TRACE(105 + kc, it);
       if (!(ok = wwait(slot_bar(ctl, k), (it & 1u) ^ 1u, ctl, kSiteDqSlot, p.dev_err))) break;
       if (lane == 0) QMLA_TRACE(88 + warp, it);  // (overwritten per chunk: last slot wait)

@@ -202,7 +202,7 @@ def test_serving_mix_256_steps():
     seqs = [0, 77, 127]
     for step in range(w.steps):
         c.append_step(step)
-        if step in (0, 1, 128, w.steps - 1):
+        if step % 32 == 0 or step in (1, w.steps - 1):  # 10 of the 256 steps, spread over the run
             out, lse = c.decode(step)
             check(c, step, seqs, out, lse)
     assert c.dev_error() == 0
