@@ -48,8 +48,17 @@ constexpr int kTileTokens = 128;                 // tokens per tile (M of QK)
 constexpr int kChunkBytes = kTileTokens * 128;   // 128 tokens x 64 fp16 channels
 constexpr int kNumChunks = 9;                    // 8 content chunks + RoPE-key chunk
 constexpr int kWorkers = 8;                      // warps 0..7: dequantise, softmax, epilogue
-constexpr int kMmaWarp = kWorkers;               // warp 8 issues MMAs and owns TMEM
-constexpr int kThreads = (kMmaWarp + 1) * 32;    // 288
+// Warps 8..11 each keep one thread that issues MMAs, one per SM sub-partition
+// (warp w runs on sub-partition w mod 4). A tcgen05.mma occupies its issuing
+// thread until the tensor core takes it, so a single issuer stalls the tensor
+// pipe whenever the scheduler of its sub-partition serves the busy worker
+// warps there; four issuers with their own accumulators keep it fed.
+constexpr int kIssuers = 4;
+constexpr int kThreads = (kWorkers + kIssuers) * 32;  // 384
+// S^T is accumulated in kQkParts partial sums, issuer j (< kQkParts) taking
+// the K-steps kk = j mod kQkParts of every chunk; the softmax adds them.
+constexpr int kQkParts = 2;
+static_assert(4 % kQkParts == 0 && kQkParts <= kIssuers, "QK split");
 constexpr uint64_t kWaitNs = 2000000000ull;      // bound of every on-chip wait (2 s)
 constexpr float kRescaleLog2 = 8.0f;             // rescale O only above 2^8 growth
 constexpr float kLn2 = 0.6931471805599453f;
@@ -117,14 +126,15 @@ struct Params {
 
 struct __align__(16) Ctrl {
   // chunk_full[k]: chunk k of the current tile is written (one arrive per warp of its parity).
-  // slot_free[j]: PV block j (chunks 2j, 2j+1) of the previous tile has completed.
-  // pv_done: a tile's whole PV has completed: chunks 6, 7 and the P tile (chunk 8's
-  // slot) are free and O^T holds the sum through that tile.
+  // pv_done: a tile's whole PV has completed (one commit per issuer, each its
+  // 128-channel block): every chunk slot and the P tile are free and O^T holds
+  // the sum through that tile.
   uint64_t chunk_full[kNumChunks];
-  uint64_t slot_free[3];
+  uint64_t pv_done;
+  // s_full: every partial of S^T is complete (one commit per QK issuer).
   // p_full: every worker wrote its part of P (one arrive per warp). p_fixed: after a
   // rescale, P was rewritten against the raised reference.
-  uint64_t pv_done, s_full, p_full, p_fixed, o_free, q_full, fin;
+  uint64_t s_full, p_full, p_fixed, o_free, q_full, fin;
   uint64_t grp;  // barrier among the worker warps (one arrive per warp, reused in sequence)
   uint32_t tmem_base;
   uint32_t abort;
@@ -141,9 +151,9 @@ static_assert(sizeof(Ctrl) % 16 == 0, "Ctrl size");
 template <int HG>
 struct Cfg {
   static constexpr int kQBytes = kNumChunks * HG * 128;
-  // O^T (4 HG columns) and S^T (HG), rounded up to a power of 2.
+  // O^T (4 HG columns) and the kQkParts partials of S^T (HG each), rounded up to a power of 2.
   static constexpr uint32_t kTmemCols = HG >= 64 ? 512 : (HG == 32 ? 256 : 128);
-  static_assert(HG > 64 || 5 * HG <= static_cast<int>(kTmemCols), "TMEM columns");
+  static_assert(HG > 64 || (4 + kQkParts) * HG <= static_cast<int>(kTmemCols), "TMEM columns");
   static constexpr int kSmem = 1024 + kNumChunks * kChunkBytes + kQBytes + (int)sizeof(Ctrl);
   static constexpr uint32_t kPRowBytes = 2 * HG;  // P^T tile row (one token, HG fp16)
 };
@@ -697,9 +707,6 @@ struct Cols {
   static_assert(kN * kW == kPerWarp, "column split");
 };
 
-// The slot of chunk k is freed by PV block k / 2 of the previous tile; the
-// RoPE chunk 8 holds that tile's P and is freed by the whole PV.
-__device__ __forceinline__ uint64_t* slot_bar(Ctrl& c, int k) { return k < 6 ? &c.slot_free[k >> 1] : &c.pv_done; }
 
 // Sum over the warp's 32 lanes of each of W values; lane l returns the total
 // of element l >> 1 (W = 16) or l >> 2 (W = 8), by recursive halving.
@@ -733,6 +740,28 @@ __device__ __forceinline__ float ex2_approx(float x) {
 // heads of earlier query tokens do not see the last positions: Eq. mla_compact's
 // causal mask, see row_limit).
 
+// W columns of this thread's row of S^T starting at t_s: the sum of the
+// kQkParts partials (HG columns apart), added in a fixed order.
+template <int HG, int W>
+__device__ __forceinline__ void load_s(uint32_t t_s, uint32_t (&r)[W]) {
+  tmem_ld(t_s, r);
+  if constexpr (kQkParts > 1) {
+    uint32_t a[kQkParts - 1][W];
+#pragma unroll
+    for (int q = 1; q < kQkParts; ++q) tmem_ld(t_s + q * HG, a[q - 1]);
+    tmem_ld_wait();
+#pragma unroll
+    for (int jj = 0; jj < W; ++jj) {
+      float v = __uint_as_float(r[jj]);
+#pragma unroll
+      for (int q = 1; q < kQkParts; ++q) v += __uint_as_float(a[q - 1][jj]);
+      r[jj] = __float_as_uint(v);
+    }
+  } else {
+    tmem_ld_wait();
+  }
+}
+
 // Tile max of the scaled scores of this warp's heads over its 32 rows into red_q[h].
 template <int HG>
 __device__ __forceinline__ void warp_tile_max(uint32_t t_s, float sl2, int lim, float* red_q, int lane) {
@@ -740,8 +769,7 @@ __device__ __forceinline__ void warp_tile_max(uint32_t t_s, float sl2, int lim, 
 #pragma unroll
   for (int c = 0; c < C::kN; ++c) {
     uint32_t r[C::kW];
-    tmem_ld(t_s + c * C::kW, r);
-    tmem_ld_wait();
+    load_s<HG>(t_s + c * C::kW, r);
 #pragma unroll
     for (int jj = 0; jj < C::kW; ++jj) {
       const float x = c * C::kW + jj >= lim ? __uint_as_float(r[jj]) * sl2 : -INFINITY;
@@ -761,8 +789,6 @@ __device__ __forceinline__ bool compute_p(uint32_t t_s, const float* mr, float s
   bool over = false;
 #pragma unroll
   for (int c = 0; c < C::kN; ++c) {
-    uint32_t r[C::kW];
-    tmem_ld(t_s + c * C::kW, r);
     float m[C::kW];
 #pragma unroll
     for (int v4 = 0; v4 < C::kW / 4; ++v4) {
@@ -772,7 +798,8 @@ __device__ __forceinline__ bool compute_p(uint32_t t_s, const float* mr, float s
       m[4 * v4 + 2] = mv.z;
       m[4 * v4 + 3] = mv.w;
     }
-    tmem_ld_wait();
+    uint32_t r[C::kW];
+    load_s<HG>(t_s + c * C::kW, r);
 #pragma unroll
     for (int jj = 0; jj < C::kW; jj += 2) {
       const float x0 = __uint_as_float(r[jj]) * sl2 - m[jj];
@@ -1007,21 +1034,26 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     const RowRef ref_nn = row_ref(p, nn, row);
     if (lane == 0 && warp == 0) QMLA_TRACE(0, it);
 
-    // ---- dequantise this tile, chunk by chunk as the previous PV frees the slots
-    // (this library's INT4 / INT2 block, protected rows included: each row's
-    // chunk computed before its slot wait; measured no faster for the paper's page)
+    // ---- dequantise this tile. The previous tile's four PV blocks (one issuer
+    // each) complete together, so one wait frees every slot. For this
+    // library's INT4 / INT2 block (protected rows included) the first chunk's
+    // arithmetic runs before that wait and each further chunk's while the
+    // stores of the one before drain, ahead of its proxy fence.
     constexpr bool kEarly = CB == 4 || CB == 2;
+    uint32_t dq[kEarly ? 32 : 1];
+    if constexpr (kEarly) row_regs<CB, PROT>(dq, f[0], par, psrc_cur);
+    if (lane == 0 && warp == 0) QMLA_TRACE(105, it);
+    if (!(ok = wwait(&ctl.pv_done, (it & 1u) ^ 1u, ctl, kSiteDqSlot, p.dev_err))) break;
+    if (lane == 0) QMLA_TRACE(88 + warp, it);
+    if (lane == 0 && (warp & 3) == 0) QMLA_TRACE(warp == 0 ? 96 : 101, it);
 #pragma unroll
     for (int kc = 0; kc < kMyChunks; ++kc) {
       const int k = 2 * kc + par;
       if (k >= kNumChunks) break;
-      uint32_t dq[kEarly ? 32 : 1];
-      if constexpr (kEarly) row_regs<CB, PROT>(dq, f[kc], k, psrc_cur);
-      if (lane == 0 && warp == 0) QMLA_TRACE(105 + kc, it);
-      if (!(ok = wwait(slot_bar(ctl, k), (it & 1u) ^ 1u, ctl, kSiteDqSlot, p.dev_err))) break;
-      if (lane == 0) QMLA_TRACE(88 + warp, it);  // (overwritten per chunk: last slot wait)
-      if (lane == 0 && (warp & 3) == 0) QMLA_TRACE((warp == 0 ? 96 : 101) + kc, it);
       if constexpr (CB == 16) {
+        // (a wait per chunk, as a scheduling barrier: without it the compiler
+        // hoists the loads of later chunks and spills)
+        if (kc > 0 && !(ok = wwait(&ctl.pv_done, (it & 1u) ^ 1u, ctl, kSiteDqSlot, p.dev_err))) break;
         uint4 nxt[8];
         const int kn = k + 2;
         const bool same = kn < kNumChunks;  // the next chunk of this tile, else the next tile's first
@@ -1032,22 +1064,28 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
         bf16_store_t(chunks + k * kChunkBytes, q4 * 32, cur, lane);
 #pragma unroll
         for (int i = 0; i < 8; ++i) cur[i] = nxt[i];
+      } else if constexpr (kEarly) {
+        store_regs(chunks + k * kChunkBytes, row, dq);
+        if (kc + 1 < kMyChunks && k + 2 < kNumChunks) row_regs<CB, PROT>(dq, f[kc + 1], k + 2, psrc_cur);
       } else {
-        if constexpr (kEarly) {
-          store_regs(chunks + k * kChunkBytes, row, dq);
-        } else {
-          dq_row<CB, PROT>(chunks + k * kChunkBytes, row, k, psrc_cur, f[kc]);
-          f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);  // the next tile's rows of this chunk
-        }
+        dq_row<CB, PROT>(chunks + k * kChunkBytes, row, k, psrc_cur, f[kc]);
+        f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);  // the next tile's rows of this chunk
       }
       fence_proxy_async_smem();
       __syncwarp();
       mbar_arrive_if(lane == 0 ? 1u : 0u, &ctl.chunk_full[k]);
-      // (the early path fetches the next tile's rows of this chunk after the arrive)
-      if constexpr (kEarly) f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);
       if (lane == 0) QMLA_TRACE(48 + warp * 5 + kc, it);
     }
     if (!ok) break;
+    if constexpr (kEarly) {
+      // The next tile's packed rows, issued once this tile's stores are out
+      // (inside the chunk loop their issue queued behind the stores).
+#pragma unroll
+      for (int kc = 0; kc < kMyChunks; ++kc) {
+        const int k = 2 * kc + par;
+        if (k < kNumChunks) f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);
+      }
+    }
     if (lane == 0) QMLA_TRACE(32 + warp, it);
     blk_cur = blk_nx;
     valid_cur = valid_nx;
@@ -1057,7 +1095,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     const TileInfo ti = tile_info(sc, p);  // ntok of this tile for the softmax
     const int lim = row_limit<HG>(p, ti, row, cb0);
 
-    // ---- the previous segment's results (its last PV completed: chunks 6..8 were waited for)
+    // ---- the previous segment's results (its last PV completed: pv_done was waited for above)
     if (pending) {
       tc_fence_after();
       if (!(ok = epilogue<CB, HG>(p, pend, ctl, tmem, gph, lsum_done, warp, lane))) break;
@@ -1184,88 +1222,95 @@ __device__ __forceinline__ void issue_query(const Params& p, int unit, uint8_t* 
   for (int k = 0; k < kNumChunks; ++k) bulk_g2s(qsmem + k * HG * 128, src + k * HG * 128, HG * 128, &ctl.q_full);
 }
 
-// Bounded wait of the single MMA thread (no warp-collective operations: the
+// Bounded wait of an MMA-issuing thread (no warp-collective operations: the
 // other lanes of its warp have exited).
 __device__ __forceinline__ bool twait(uint64_t* bar, uint32_t parity, Ctrl& c, uint32_t site, uint32_t* dev_err) {
   return wait_ok(mbar_wait(bar, parity, kWaitNs, &c.abort), site, c, dev_err);
 }
 
-// One thread issues every MMA, commit and query copy (the other lanes of its
-// warp exit at the start: a warp whose lane 0 issues or waits while the other
-// lanes sit at a re-convergence point was measured to issue MMAs and wake up
-// far more slowly on sm_103a). A commit tracks the MMAs issued by the
-// committing thread. QK starts on each chunk as soon as it is written; PV
-// commits after each 128-channel block so that the next tile's
-// dequantisation can refill those slots. Descriptors are advanced by adding
-// (byte offset >> 4) to their start-address field.
+// Issuer j (0..3, one thread of warp 8 + j; the other lanes exit at the start:
+// a warp whose lane 0 issues or waits while the other lanes sit at a
+// re-convergence point was measured to issue MMAs and wake up far more slowly
+// on sm_103a) issues K-steps kk = j mod kQkParts of every QK chunk into S^T
+// partial j, and PV block j (channels 128 j .. 128 j + 127) into O^T block j.
+// A commit tracks the MMAs issued by the committing thread, so each issuer
+// commits its own: s_full counts the QK partials, pv_done the PV blocks. Issuer 0 also copies the query
+// images. QK starts on each chunk as soon as it is written. Descriptors are
+// advanced by adding (byte offset >> 4) to their start-address field.
 template <int HG>
-__device__ void mma_thread(const Params& p, Sched sc, uint32_t chunks, uint8_t* qsmem, Ctrl& ctl, uint32_t tmem) {
+__device__ void mma_issuer(const Params& p, Sched sc, uint32_t chunks, uint8_t* qsmem, Ctrl& ctl, uint32_t tmem,
+                           int j) {
   constexpr uint32_t kIdQK = idesc_f16_f32(128, HG, false, false);
   constexpr uint32_t kIdPV = idesc_f16_f32(128, HG, true, true);
   constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
   constexpr uint32_t kSboP = 8 * kRB;
+  constexpr int kSteps = 4 / kQkParts;  // QK K-steps per chunk and issuer
+  const bool qk = j < kQkParts;
   const uint32_t qbase = smem_u32(qsmem);
   const uint32_t ptile = chunks + 8 * kChunkBytes;
-  const uint32_t t_s = tmem + 4 * HG;
-  const uint64_t qk_a0 = smem_desc(chunks, 16, 1024, SWZ_128B);
-  const uint64_t qk_b0 = smem_desc(qbase, 16, 1024, SWZ_128B);
-  const uint64_t pv_a0 = smem_desc(chunks, kChunkBytes, 1024, SWZ_128B);
+  const uint32_t t_s = tmem + (4 + j) * HG;  // S^T partial j
+  const uint32_t t_o = tmem + j * HG;        // O^T block j
+  const uint64_t qk_a0 = smem_desc(chunks, 16, 1024, SWZ_128B) + static_cast<uint64_t>((j * 32) >> 4);
+  const uint64_t qk_b0 = smem_desc(qbase, 16, 1024, SWZ_128B) + static_cast<uint64_t>((j * 32) >> 4);
+  const uint64_t pv_a0 =
+      smem_desc(chunks, kChunkBytes, 1024, SWZ_128B) + static_cast<uint64_t>((2 * j * kChunkBytes) >> 4);
   const uint64_t pv_b0 = smem_desc(ptile, 16 * kSboP, kSboP, swz_mode_for_row(kRB));
   uint32_t it = 0, seg = 0, nresc = 0;
   bool ok = true;
-  if (sc.valid()) issue_query<HG>(p, sc.u, qsmem, ctl);
+  if (j == 0 && sc.valid()) issue_query<HG>(p, sc.u, qsmem, ctl);
   for (; ok && sc.valid(); sc.next()) {
     const TileFlags ti = tile_flags(sc);
-    QMLA_TRACE(1, it);
+    if (j == 0) QMLA_TRACE(1, it);
     if (ti.first && !(ok = twait(&ctl.q_full, seg & 1u, ctl, kSiteMmaQFull, p.dev_err))) break;
-    // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576), chunk by
-    // chunk. The next chunk's barrier is probed before this chunk's MMAs are
-    // issued, so the probe's latency overlaps them; only a chunk that was not
-    // yet written takes the (bounded) wait.
-    // (Unrolled by three: fully unrolled, the first tile after a cold start
-    // spends thousands of cycles fetching the loop's instructions.)
-    bool ready = mbar_test(&ctl.chunk_full[0], it & 1u);
+    if (qk) {
+      // S^T = C_hat . q^T over the nine 64-channel chunks (K = 576), chunk by
+      // chunk. The next chunk's barrier is probed before this chunk's MMAs are
+      // issued, so the probe's latency overlaps them; only a chunk that was not
+      // yet written takes the (bounded) wait.
+      // (Unrolled by three: fully unrolled, the first tile after a cold start
+      // spends thousands of cycles fetching the loop's instructions.)
+      bool ready = mbar_test(&ctl.chunk_full[0], it & 1u);
 #pragma unroll 3
-    for (int k = 0; k < kNumChunks; ++k) {
-      if (!ready && !(ok = twait(&ctl.chunk_full[k], it & 1u, ctl, kSiteMmaChunk, p.dev_err))) break;
-      tc_fence_after();
-      QMLA_TRACE(112 + k, it);
-      if (k + 1 < kNumChunks) ready = mbar_test(&ctl.chunk_full[k + 1], it & 1u);
+      for (int k = 0; k < kNumChunks; ++k) {
+        if (!ready && !(ok = twait(&ctl.chunk_full[k], it & 1u, ctl, kSiteMmaChunk, p.dev_err))) break;
+        tc_fence_after();
+        if (j == 0) QMLA_TRACE(112 + k, it);
+        if (k + 1 < kNumChunks) ready = mbar_test(&ctl.chunk_full[k + 1], it & 1u);
 #pragma unroll
-      for (int kk = 0; kk < 4; ++kk)
-        umma_f16_ss(t_s, qk_a0 + static_cast<uint64_t>((k * kChunkBytes + kk * 32) >> 4),
-                    qk_b0 + static_cast<uint64_t>((k * HG * 128 + kk * 32) >> 4), kIdQK, (k | kk) != 0 ? 1u : 0u);
+        for (int kk = 0; kk < kSteps; ++kk)
+          umma_f16_ss(t_s, qk_a0 + static_cast<uint64_t>((k * kChunkBytes + kk * kQkParts * 32) >> 4),
+                      qk_b0 + static_cast<uint64_t>((k * HG * 128 + kk * kQkParts * 32) >> 4), kIdQK,
+                      (k | kk) != 0 ? 1u : 0u);
+      }
+      if (!ok) break;
+      umma_commit(&ctl.s_full);
     }
-    if (!ok) break;
-    umma_commit(&ctl.s_full);
-    QMLA_TRACE(12, it);
+    if (j == 0) QMLA_TRACE(12, it);
     if (!(ok = twait(&ctl.p_full, it & 1u, ctl, kSiteMmaPFull, p.dev_err))) break;
     if (*reinterpret_cast<volatile uint32_t*>(&ctl.resc_tile) == it + 1) {
       if (!(ok = twait(&ctl.p_fixed, nresc & 1u, ctl, kSiteMmaPFull, p.dev_err))) break;
       ++nresc;
     }
-    QMLA_TRACE(14, it);
-    if (ti.last) {
-      // The softmax only signals P after this tile's QK has completed, so the
-      // query tile is free: start copying the next segment's query now.
+    if (j == 0) QMLA_TRACE(14, it);
+    if (j == 0 && ti.last) {
+      // The softmax only signals P after every QK partial of this tile has
+      // completed, so the query tile is free: start copying the next
+      // segment's query now.
       Sched nx = sc;
       nx.next();
       if (nx.valid()) issue_query<HG>(p, nx.u, qsmem, ctl);
     }
     if (ti.first && seg > 0 && !(ok = twait(&ctl.o_free, (seg - 1) & 1u, ctl, kSiteMmaOFree, p.dev_err))) break;
     tc_fence_after();
-    // O^T[c, h] += sum_t C_hat[t, c] P^T[t, h], 4 x 128 channels, K = 128 tokens.
+    // O^T[c, h] += sum_t C_hat[t, c] P^T[t, h] for this issuer's 128 channels, K = 128 tokens.
     const uint32_t acc0 = ti.first ? 0u : 1u;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-#pragma unroll
-      for (int kk = 0; kk < 8; ++kk)
-        umma_f16_ss(tmem + i * HG, pv_a0 + static_cast<uint64_t>((2 * i * kChunkBytes + kk * 2048) >> 4),
-                    pv_b0 + static_cast<uint64_t>((kk * 2 * kSboP) >> 4), kIdPV, kk == 0 ? acc0 : 1u);
-      umma_commit(i < 3 ? &ctl.slot_free[i] : &ctl.pv_done);
-      QMLA_TRACE(24 + i, it);
-    }
-    QMLA_TRACE(15, it);
+    for (int kk = 0; kk < 8; ++kk)
+      umma_f16_ss(t_o, pv_a0 + static_cast<uint64_t>((kk * 2048) >> 4),
+                  pv_b0 + static_cast<uint64_t>((kk * 2 * kSboP) >> 4), kIdPV, kk == 0 ? acc0 : 1u);
+    umma_commit(&ctl.pv_done);
+    QMLA_TRACE(24 + j, it);
+    if (j == 0) QMLA_TRACE(15, it);
     ++it;
     if (ti.last) ++seg;
   }
@@ -1295,15 +1340,14 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
 
   if (threadIdx.x == 0) {
     for (int k = 0; k < kNumChunks; ++k) mbar_init(&ctl.chunk_full[k], 4);
-    for (int j = 0; j < 3; ++j) mbar_init(&ctl.slot_free[j], 1);
-    mbar_init(&ctl.pv_done, 1);
-    mbar_init(&ctl.s_full, 1);
+    mbar_init(&ctl.pv_done, kIssuers);
+    mbar_init(&ctl.s_full, kQkParts);
     mbar_init(&ctl.p_full, kWorkers);
     mbar_init(&ctl.p_fixed, kWorkers);
     ctl.resc_tile = 0u;
     mbar_init(&ctl.o_free, kWorkers);
     mbar_init(&ctl.q_full, 1);
-    mbar_init(&ctl.fin, 1);
+    mbar_init(&ctl.fin, kIssuers);
     mbar_init(&ctl.grp, kWorkers);
     ctl.abort = 0u;
     fence_mbar_init();
@@ -1316,7 +1360,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = ctl.tmem_base;
-  if (warp == kMmaWarp && lane != 0) return;  // the MMA role is a single thread
+  if (warp >= kWorkers && lane != 0) return;  // each MMA role is a single thread
   // The set-up above may overlap the prep kernel; everything below reads what
   // prep and the cache writer before it produced.
   griddep_wait();
@@ -1326,11 +1370,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   if (warp < kWorkers) {
     worker_role<CB, HG, PROT>(p, sc, chunks, ctl, tmem, warp, lane);
   } else {
-    mma_thread<HG>(p, sc, chunks, qsmem, ctl, tmem);
+    mma_issuer<HG>(p, sc, chunks, qsmem, ctl, tmem, warp - kWorkers);
   }
   griddep_launch_dependents();  // the merge may be scheduled as CTAs finish
   tc_fence_before();
-  __syncthreads();  // the exited lanes of the MMA warp do not take part
+  __syncthreads();  // the exited lanes of the MMA warps do not take part
   if (warp == 0) {
     tc_fence_after();
     tmem_dealloc(tmem, Cfg<HG>::kTmemCols);
