@@ -100,7 +100,9 @@ size_t qmla_bf16_block_bytes(void);
  * (App. C.4 quantiser; App. C.5 fused writer without the BF16 protection
  * buffers).
  *
- *   pool_dev        [num_blocks * qmla_block_bytes(c_bits)] bytes, 16-byte aligned;
+ *   pool_dev        [num_blocks * qmla_block_bytes(c_bits)] bytes, 32-byte aligned
+ *                   (every call that takes a pool requires this: the decode
+ *                   reads a token's 32-byte code row in one request);
  *                   only the slots of the given tokens are written
  *   c_bits          content bit width, 4 or 2 (the RoPE key is always 4-bit)
  *   latent_dev      [n, 512] bf16, row-major, 4-byte aligned: content latent c_KV
@@ -170,7 +172,8 @@ size_t qmla_decode_workspace_bytes(int batch, int heads);
  * The caller applies the value/output up-projection. Sequences are split
  * across the GPU's SMs and the split results merged with the App. C.5 rule.
  *
- *   pool_dev        packed cache written by qmla_quant_append with the same c_bits
+ *   pool_dev        packed cache written by qmla_quant_append with the same c_bits,
+ *                   32-byte aligned
  *   q_latent_dev    [batch, heads, 512] bf16 absorbed content query, 16-byte aligned
  *   q_pe_dev        [batch, heads, 64]  bf16 RoPE query, 16-byte aligned
  *   heads           1..128

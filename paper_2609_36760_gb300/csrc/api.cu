@@ -50,7 +50,7 @@ int append_common_checks(const void* pool, int num_blocks, const uint16_t* laten
   if (n == 0) return QMLA_OK;
   if (pool == nullptr || latent == nullptr || k_pe == nullptr || positions == nullptr || table == nullptr)
     return QMLA_ERR_INVALID_ARG;
-  if (!aligned(pool, 16) || !aligned(latent, 4) || !aligned(k_pe, 4) || !aligned(positions, 4) ||
+  if (!aligned(pool, 32) || !aligned(latent, 4) || !aligned(k_pe, 4) || !aligned(positions, 4) ||
       !aligned(table, 4))
     return QMLA_ERR_INVALID_ARG;
   if (static_cast<long long>(max_blocks) * qmla::kBlockTokens > INT32_MAX) return QMLA_ERR_INVALID_ARG;
@@ -71,7 +71,7 @@ int decode_checks(const void* pool, int num_blocks, const uint16_t* q_latent, co
   if (batch <= 0 || heads < 1 || heads / q_tokens > 128 || num_blocks <= 0 || max_blocks <= 0)
     return QMLA_ERR_INVALID_ARG;
   if (!(softmax_scale > 0.0f) || softmax_scale > 1e30f) return QMLA_ERR_INVALID_ARG;
-  if (!aligned(pool, 16) || !aligned(q_latent, 16) || !aligned(q_pe, 16) || !aligned(table, 4) ||
+  if (!aligned(pool, 32) || !aligned(q_latent, 16) || !aligned(q_pe, 16) || !aligned(table, 4) ||
       !aligned(seq_lens, 4) || !aligned(out, 16) || (lse != nullptr && !aligned(lse, 4)) ||
       (need_workspace && !aligned(workspace, 256)))
     return QMLA_ERR_INVALID_ARG;
@@ -304,7 +304,7 @@ int qmla_debug_tile(const void* pool_dev, int cache_kind, int num_blocks, const 
   if (num_blocks <= 0 || max_blocks <= 0 || batch <= 0 || b < 0 || b >= batch || j < 0 ||
       static_cast<long long>(j) * 2 >= max_blocks)
     return QMLA_ERR_INVALID_ARG;
-  if (!aligned(pool_dev, 16) || !aligned(tile_dev, 16) || (prot_dev != nullptr && !aligned(prot_dev, 16)))
+  if (!aligned(pool_dev, 32) || !aligned(tile_dev, 16) || (prot_dev != nullptr && !aligned(prot_dev, 16)))
     return QMLA_ERR_INVALID_ARG;
   if (prot_dev != nullptr && cache_kind == QMLA_CACHE_BF16) return QMLA_ERR_INVALID_ARG;
   DevInfo di;

@@ -186,6 +186,12 @@ __device__ __forceinline__ uint4 ldg_nc_v4(const void* ptr) {
                : "l"(ptr));
   return r;
 }
+// 32 bytes in one request (the address is 32-byte aligned).
+__device__ __forceinline__ void ldg_nc_v8(const void* ptr, uint4& a, uint4& b) {
+  asm volatile("ld.global.nc.L1::no_allocate.v8.u32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+               : "=r"(a.x), "=r"(a.y), "=r"(a.z), "=r"(a.w), "=r"(b.x), "=r"(b.y), "=r"(b.z), "=r"(b.w)
+               : "l"(ptr));
+}
 __device__ __forceinline__ uint32_t ldg_nc_u32(const void* ptr) {
   uint32_t r;
   asm volatile("ld.global.nc.L1::no_allocate.u32 %0, [%1];" : "=r"(r) : "l"(ptr));
@@ -399,8 +405,13 @@ __device__ __forceinline__ Fetch fetch_chunk(const uint8_t* blk, bool valid, int
   if (!valid) return f;
   using L = BlockLayout<CB>;
   const uint8_t* c = blk + L::code_off(k, slot);
-  f.a = ldg_nc_v4(c);
-  if (CB == 4 || CB == kC4R4 || k == 8) f.b = ldg_nc_v4(c + 16);
+  // a 32-byte code row in one request (half the requests of two 16-byte
+  // loads, which made the next tile's fetch a quarter of the kernel's time)
+  if (CB == 4 || CB == kC4R4 || k == 8) {
+    ldg_nc_v8(c, f.a, f.b);
+  } else {
+    f.a = ldg_nc_v4(c);
+  }
   if constexpr (CB == kC4R4) {
     // bf16 content scale -> fp32 bits by a 16-bit shift; the RoPE scale is fp32
     f.sz = k < 8 ? ldg_nc_u16(blk + L::c_scale_off(k, slot)) << 16 : ldg_nc_u32(blk + L::pe_scale_off(slot));
@@ -408,6 +419,24 @@ __device__ __forceinline__ Fetch fetch_chunk(const uint8_t* blk, bool valid, int
   } else {
     f.sz = ldg_nc_u32(blk + L::sz_off(k, slot));
   }
+  return f;
+}
+
+// Half h of a token row of the RoPE-key chunk (INT4 codes of channels 32 h ..
+// 32 h + 31, bytes 16 h .. 16 h + 15): the two worker warps that share a row
+// quarter split that chunk, so each dequantises 4.5 chunks per tile.
+template <int CB>
+__device__ __forceinline__ Fetch fetch_rope_half(const uint8_t* blk, bool valid, int slot, int h) {
+  Fetch f;
+  f.ok = valid;
+  f.a = make_uint4(0, 0, 0, 0);
+  f.b = f.a;
+  f.sz = 0;
+  f.z = 0;
+  if (!valid) return f;
+  using L = BlockLayout<CB>;
+  f.a = ldg_nc_v4(blk + L::code_off(8, slot) + 16 * h);
+  f.sz = ldg_nc_u32(blk + L::sz_off(8, slot));
   return f;
 }
 
@@ -492,6 +521,31 @@ __device__ __forceinline__ void store_regs(uint32_t chunk_base, int row, const u
 #pragma unroll
   for (int i = 0; i < 8; ++i)
     sts_v4(chunk_base + swz_off(row, i, 128), o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
+}
+// Half h of a RoPE-key row (fetch_rope_half): o[0..15] from the 32 INT4 codes
+// of f.a, the same arithmetic as dq_regs; stored as pieces 4 h .. 4 h + 3.
+__device__ __forceinline__ void dq_half(uint32_t (&o)[32], const Fetch& f) {
+  const __half2 sz = *reinterpret_cast<const __half2*>(&f.sz);
+  const __half2 s2 = __half2half2(__low2half(sz));
+  const __half2 zz2 = __half2half2(__hadd(__high2half(sz), __float2half_rn(1024.0f)));
+  const uint32_t ss = *reinterpret_cast<const uint32_t*>(&s2);
+  const uint32_t zz = *reinterpret_cast<const uint32_t*>(&zz2);
+  constexpr uint32_t K = 0x64646464u;
+  const uint32_t w[4] = {f.a.x, f.a.y, f.a.z, f.a.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t lo = w[i] & 0x0F0F0F0Fu;
+    const uint32_t hi = (w[i] >> 4) & 0x0F0F0F0Fu;
+    o[4 * i + 0] = dq2(__byte_perm(lo, K, 0x4140), zz, ss);
+    o[4 * i + 1] = dq2(__byte_perm(hi, K, 0x4140), zz, ss);
+    o[4 * i + 2] = dq2(__byte_perm(lo, K, 0x4342), zz, ss);
+    o[4 * i + 3] = dq2(__byte_perm(hi, K, 0x4342), zz, ss);
+  }
+}
+__device__ __forceinline__ void store_half(uint32_t chunk_base, int row, const uint32_t (&o)[32], int h) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    sts_v4(chunk_base + swz_off(row, 4 * h + i, 128), o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
 }
 
 // Rows of the paper's page. store_row_c4r4 writes one row (64 INT4 codes) of
@@ -629,6 +683,33 @@ __device__ __forceinline__ void row_regs(uint32_t (&o)[32], const Fetch& f, int 
   // hoisted above the arithmetic.
 #pragma unroll
   for (int i = 0; i < 32; ++i) asm volatile("" : "+r"(o[i]));
+}
+// Half h of a RoPE-key row into o[0..15] (pieces 4 h .. 4 h + 3): the
+// protection row's bf16 channels 32 h .. 32 h + 31 rounded to fp16 when the
+// row is protected, else dq_half of the packed codes.
+template <bool PROT>
+__device__ __forceinline__ void row_regs_half(uint32_t (&o)[32], const Fetch& f, const uint8_t* ps, int h) {
+  if (PROT && ps != nullptr) {
+    uint4 pv[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) pv[i] = __ldg(reinterpret_cast<const uint4*>(ps + 8 * 128 + h * 64) + i);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const uint32_t w[4] = {pv[i].x, pv[i].y, pv[i].z, pv[i].w};
+      float v[8];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        v[2 * e] = bf16_lo(w[e]);
+        v[2 * e + 1] = bf16_hi(w[e]);
+      }
+#pragma unroll
+      for (int e = 0; e < 4; ++e) o[4 * i + e] = pack_h2(v[Perm<4>::at(2 * e)], v[Perm<4>::at(2 * e + 1)]);
+    }
+  } else {
+    dq_half(o, f);
+  }
+#pragma unroll
+  for (int i = 0; i < 16; ++i) asm volatile("" : "+r"(o[i]));
 }
 
 // BF16 cache rows read coalesced: lane l of a warp handles piece l & 7 (16
@@ -949,7 +1030,10 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
   const uint32_t t_o = tmem + cb0 + lane_off;
   const uint32_t ptile = chunks + 8 * kChunkBytes;
   const float sl2 = p.scale_log2;
-  constexpr int kMyChunks = 5;  // chunks per parity, rounded up (parity 1 has 4)
+  constexpr int kMyChunks = 5;  // chunk steps per warp (the paper's page and BF16: parity 1 has 4)
+  // This library's INT4 / INT2 block: each warp dequantises 4 content chunks
+  // and half of the RoPE-key chunk (channels 32 par .. 32 par + 31).
+  constexpr bool kEarly = CB == 4 || CB == 2;
   uint32_t it = 0, gph = 0, nresc = 0;
   int seg_j0 = 0;
   bool ok = true;
@@ -984,7 +1068,11 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     }
   }
   const uint8_t* blk_cur = psrc_cur != nullptr ? nullptr : resolve_row<CB>(p, ref0, row, valid_cur);
-  if constexpr (CB != 16) {
+  if constexpr (kEarly) {
+#pragma unroll
+    for (int kc = 0; kc < 4; ++kc) f[kc] = fetch_chunk<CB>(blk_cur, valid_cur, 2 * kc + par, slot);
+    f[4] = fetch_rope_half<CB>(blk_cur, valid_cur, slot, par);
+  } else if constexpr (CB != 16) {
 #pragma unroll
     for (int kc = 0; kc < kMyChunks; ++kc) {
       const int k = 2 * kc + par;
@@ -1039,7 +1127,6 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     // library's INT4 / INT2 block (protected rows included) the first chunk's
     // arithmetic runs before that wait and each further chunk's while the
     // stores of the one before drain, ahead of its proxy fence.
-    constexpr bool kEarly = CB == 4 || CB == 2;
     uint32_t dq[kEarly ? 32 : 1];
     if constexpr (kEarly) row_regs<CB, PROT>(dq, f[0], par, psrc_cur);
     if (lane == 0 && warp == 0) QMLA_TRACE(105, it);
@@ -1048,7 +1135,8 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     if (lane == 0 && (warp & 3) == 0) QMLA_TRACE(warp == 0 ? 96 : 101, it);
 #pragma unroll
     for (int kc = 0; kc < kMyChunks; ++kc) {
-      const int k = 2 * kc + par;
+      // (this library's block: content chunks 2 kc + par, then half par of the RoPE chunk)
+      const int k = kEarly && kc == 4 ? 8 : 2 * kc + par;
       if (k >= kNumChunks) break;
       if constexpr (CB == 16) {
         // (a wait per chunk, as a scheduling barrier: without it the compiler
@@ -1065,8 +1153,17 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
 #pragma unroll
         for (int i = 0; i < 8; ++i) cur[i] = nxt[i];
       } else if constexpr (kEarly) {
-        store_regs(chunks + k * kChunkBytes, row, dq);
-        if (kc + 1 < kMyChunks && k + 2 < kNumChunks) row_regs<CB, PROT>(dq, f[kc + 1], k + 2, psrc_cur);
+        if (kc < 4) {
+          store_regs(chunks + k * kChunkBytes, row, dq);
+        } else {
+          store_half(chunks + 8 * kChunkBytes, row, dq, par);
+        }
+        // the next chunk's arithmetic while these stores drain
+        if (kc + 1 < 4) {
+          row_regs<CB, PROT>(dq, f[kc + 1], k + 2, psrc_cur);
+        } else if (kc + 1 == 4) {
+          row_regs_half<PROT>(dq, f[4], psrc_cur, par);
+        }
       } else {
         dq_row<CB, PROT>(chunks + k * kChunkBytes, row, k, psrc_cur, f[kc]);
         f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);  // the next tile's rows of this chunk
@@ -1081,10 +1178,8 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       // The next tile's packed rows, issued once this tile's stores are out
       // (inside the chunk loop their issue queued behind the stores).
 #pragma unroll
-      for (int kc = 0; kc < kMyChunks; ++kc) {
-        const int k = 2 * kc + par;
-        if (k < kNumChunks) f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);
-      }
+      for (int kc = 0; kc < 4; ++kc) f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, 2 * kc + par, slot);
+      f[4] = fetch_rope_half<CB>(blk_nx, valid_nx, slot, par);
     }
     if (lane == 0) QMLA_TRACE(32 + warp, it);
     blk_cur = blk_nx;
@@ -1339,7 +1434,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   }
 
   if (threadIdx.x == 0) {
-    for (int k = 0; k < kNumChunks; ++k) mbar_init(&ctl.chunk_full[k], 4);
+    // chunk k is written by the 4 warps of its parity; this library's INT4 /
+    // INT2 block splits the RoPE chunk (k = 8) over all 8 workers
+    for (int k = 0; k < kNumChunks; ++k) mbar_init(&ctl.chunk_full[k], k == 8 && (CB == 4 || CB == 2) ? 8 : 4);
     mbar_init(&ctl.pv_done, kIssuers);
     mbar_init(&ctl.s_full, kQkParts);
     mbar_init(&ctl.p_full, kWorkers);

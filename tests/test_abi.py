@@ -53,8 +53,9 @@ def test_invalid_arguments_are_rejected_before_any_launch(libqmla):
     assert L.qmla_quant_append(fake, 3, 4, fake, fake, None, fake, 1, fake, 1, 1, None, None) == 1
     # null positions
     assert L.qmla_quant_append(fake, 4, 4, fake, fake, None, None, 1, fake, 1, 1, None, None) == 1
-    # misaligned pool
+    # misaligned pool (32-byte alignment)
     assert L.qmla_quant_append(ctypes.c_void_p(0x10001), 4, 4, fake, fake, None, fake, 1, fake, 1, 1, None, None) == 1
+    assert L.qmla_quant_append(ctypes.c_void_p(0x10010), 4, 4, fake, fake, None, fake, 1, fake, 1, 1, None, None) == 1
     # n == 0 is a no-op that touches nothing
     assert L.qmla_quant_append(None, 4, 4, None, None, None, None, 0, None, 1, 1, None, None) == 0
     # decode: heads out of range, null output, bad scale, bad bits
@@ -126,7 +127,7 @@ def test_decode_ex_host_checks(libqmla):
     assert L.qmla_mla_decode_ex(None, None) == 1                       # no descriptor
     for bad in ({"cache_kind": 3}, {"cache_kind": 8}, {"q_tokens": 0}, {"q_tokens": 9}, {"heads": 0},
                 {"heads": 129}, {"batch": 0}, {"out": None}, {"workspace": None}, {"softmax_scale": -1.0},
-                {"pool": 0x10008}, {"workspace": 0x10010}, {"prot": 0x10008},
+                {"pool": 0x10008}, {"pool": 0x10010}, {"workspace": 0x10010}, {"prot": 0x10008},
                 {"cache_kind": 16, "prot": 0x10000},                     # no protection on the BF16 cache
                 {"cache_kind": 16, "q_tokens": 2}, {"cache_kind": 5, "q_tokens": 2}):
         d = _desc(**bad)
