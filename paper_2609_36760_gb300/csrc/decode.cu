@@ -1105,6 +1105,12 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       }
     }
     const uint8_t* blk_nx = psrc_nx != nullptr ? nullptr : resolve_row<CB>(p, ref_nx, row, valid_nx);
+    if constexpr (CB != 16) {
+      // The next tile's two packed blocks into L2 by the bulk-copy engine (one
+      // request each, from the threads of rows 0 and 64), so that the register
+      // fetch of its rows after this tile's chunk loop reads L2, not DRAM.
+      if (lane == 0 && (q4 & 1) == 0 && par == 0 && valid_nx) bulk_prefetch_l2(blk_nx, BlockLayout<CB>::kBytes);
+    }
     if constexpr (CB == 16) {
       // BF16 cache: its rows are read only one chunk ahead into registers, so
       // bring the next tile's lines of this thread's row and chunks into L2 now.

@@ -96,6 +96,12 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       : "memory");
 }
 
+// Asks the bulk-copy engine to bring `bytes` (a multiple of 16) at a 16-byte
+// aligned global address into L2; no completion to wait for, no registers held.
+__device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 // Orders this thread's generic-proxy shared-memory writes before later
 // async-proxy reads (tensor core operands, bulk copies).
 __device__ __forceinline__ void fence_proxy_async_smem() {
