@@ -721,12 +721,13 @@ TRACE_CTAS, TRACE_EVENTS, TRACE_TILES = 8, 128, 32
 
 def main_trace_summary(ev):
     """Median stage lengths (cycles) of decode_main's steady tiles (2 .. n-2 of
-    each traced CTA). Event numbers as stamped in decode.cu: MMA thread 112 + k
-    QK of chunk k issued, 12 QK committed, 14 P seen, 15 PV issued; worker warp
-    0: 0 loop top, 16 scores seen, 19 P written, 17 every warp's P seen, 18 row
-    sums added; lane 0 of warp w: 88 + w last slot wait passed, 32 + w tile
-    dequantised, 48 + 5 w + kc chunk step kc arrived; warp 0 (4) also 105 + kc
-    (-) chunk computed and 96 + kc (101 + kc) its slot wait passed."""
+    each traced CTA). Event numbers as stamped in decode.cu: MMA issuer 0: 1
+    loop top, 112 + k QK of chunk k issued, 12 its QK committed, 14 P seen, 15
+    its PV issued; issuer j: 24 + j its PV block committed; worker warp 0: 0
+    loop top, 105 first chunk computed, 16 scores seen, 19 P written, 17 every
+    warp's P seen, 18 row sums added; lane 0 of worker warp w: 88 + w the
+    previous PV's completion seen, 48 + 5 w + kc chunk step kc arrived, 32 + w
+    tile dequantised and the next tile's rows fetched."""
     import numpy as np
 
     stages, period = {}, []
@@ -734,19 +735,18 @@ def main_trace_summary(ev):
         n = int((ev[c, 12] > 0).sum())
         for it in range(2, n - 1):
             g, nx = ev[c, :, it], ev[c, :, it + 1]
-            period.append(nx[12] - g[12])
-            for name, v in (("mma: QK chunk 0 -> chunk 8 issued", g[120] - g[112]),
-                            ("mma: QK chunk 8 issued -> committed", g[12] - g[120]),
-                            ("mma: QK committed -> P seen", g[14] - g[12]),
-                            ("mma: P seen -> PV issued", g[15] - g[14]),
-                            ("mma: PV issued -> next QK chunk 0", nx[112] - g[15]),
-                            ("warp0: QK committed -> scores seen", g[16] - g[12]),
-                            ("warp0: scores seen -> P written", g[19] - g[16]),
-                            ("warp0: P written -> all P seen", g[17] - g[19]),
-                            ("warp0: all P seen -> row sums added", g[18] - g[17]),
-                            ("warp0: row sums added -> next loop top", nx[0] - g[18]),
-                            ("dequant: PV issued -> tile dequantised (max warp)",
-                             max(nx[32 + w] for w in range(8)) - g[15])):
+            period.append(nx[14] - g[14])
+            for name, v in (("issuer 0: QK chunk 0 -> chunk 8 issued", g[120] - g[112]),
+                            ("issuer 0: QK chunk 8 issued -> committed", g[12] - g[120]),
+                            ("issuer 0: QK committed -> P seen", g[14] - g[12]),
+                            ("issuer 0: P seen -> PV issued", g[15] - g[14]),
+                            ("issuer 0: PV issued -> next QK chunk 0", nx[112] - g[15]),
+                            ("warp 0: QK committed -> scores seen", g[16] - g[12]),
+                            ("warp 0: scores seen -> P written", g[19] - g[16]),
+                            ("warp 0: P written -> all P seen", g[17] - g[19]),
+                            ("warp 0: all P seen -> row sums added", g[18] - g[17]),
+                            ("warp 0: row sums added -> next loop top", nx[0] - g[18]),
+                            ("warp 0: loop top -> first chunk computed", nx[105] - nx[0])):
                 stages.setdefault(name, []).append(v)
     # the next tile's dequantisation relative to this tile's PV start (P seen, event 14)
     for c in range(ev.shape[0]):
@@ -754,20 +754,16 @@ def main_trace_summary(ev):
         for it in range(2, n - 1):
             g, nx = ev[c, :, it], ev[c, :, it + 1]
             t0 = g[14]
-            rel = {"mma PV block %d committed" % i: g[24 + i] - t0 for i in range(4)}
-            rel["mma PV issued"] = g[15] - t0
-            rel["mma next loop top"] = nx[1] - t0
-            for kc in range(5):
-                k = 2 * kc
-                rel["w0 chunk %d dq done" % k] = nx[105 + kc] - t0
-                rel["w0 chunk %d slot passed" % k] = nx[96 + kc] - t0
-                rel["w0 chunk %d arrived" % k] = nx[48 + kc] - t0
-            for kc in range(4):
-                k = 2 * kc + 1
-                rel["w4 chunk %d slot passed" % k] = nx[101 + kc] - t0
-                rel["w4 chunk %d arrived" % k] = nx[68 + kc] - t0
+            rel = {"issuer %d PV block committed" % j: g[24 + j] - t0 for j in range(4)}
+            for w in range(8):
+                rel["warp %d previous PV seen complete" % w] = nx[88 + w] - t0
+            for w in (0, 4):
+                for kc in range(5):
+                    rel["warp %d chunk step %d arrived" % (w, kc)] = nx[48 + 5 * w + kc] - t0
+            rel["slowest warp: tile dequantised, next rows fetched"] = max(nx[32 + w] for w in range(8)) - t0
             for k in range(9):
-                rel["mma next QK chunk %d issued" % k] = nx[112 + k] - t0
+                rel["issuer 0: next QK chunk %d issued" % k] = nx[112 + k] - t0
+            rel["issuer 0: next QK committed"] = nx[12] - t0
             for name, v in rel.items():
                 stages.setdefault("t(PV start) + " + name, []).append(v)
     if not period:
@@ -775,7 +771,7 @@ def main_trace_summary(ev):
         return
     print(f"decode_main tile period (cycles, median over {len(period)} tiles): {np.median(period):.0f}")
     for k, v in stages.items():
-        print(f"  {k:56s} {np.median(v):7.0f}")
+        print(f"  {k:60s} {np.median(v):7.0f}")
 
 
 def run_trace(args):
