@@ -131,10 +131,11 @@ struct __align__(16) Ctrl {
   // the sum through that tile.
   uint64_t chunk_full[kNumChunks];
   uint64_t pv_done;
+  // rs_done: a tile's row-sum MMAs (issued after its PV, own commit) have completed.
   // s_full: every partial of S^T is complete (one commit per QK issuer).
   // p_full: every worker wrote its part of P (one arrive per warp). p_fixed: after a
   // rescale, P was rewritten against the raised reference.
-  uint64_t s_full, p_full, p_fixed, o_free, q_full, fin;
+  uint64_t rs_done, s_full, p_full, p_fixed, o_free, q_full, fin;
   uint64_t grp;  // barrier among the worker warps (one arrive per warp, reused in sequence)
   uint32_t tmem_base;
   uint32_t abort;
@@ -151,9 +152,12 @@ static_assert(sizeof(Ctrl) % 16 == 0, "Ctrl size");
 template <int HG>
 struct Cfg {
   static constexpr int kQBytes = kNumChunks * HG * 128;
-  // O^T (4 HG columns) and the kQkParts partials of S^T (HG each), rounded up to a power of 2.
+  // O^T (4 HG columns), the kQkParts partials of S^T (HG each), the row sums
+  // of P (HG) and the all-ones A operand of their MMAs (8), rounded up to a power of 2.
   static constexpr uint32_t kTmemCols = HG >= 64 ? 512 : (HG == 32 ? 256 : 128);
-  static_assert(HG > 64 || (4 + kQkParts) * HG <= static_cast<int>(kTmemCols), "TMEM columns");
+  static constexpr uint32_t kColL = (4 + kQkParts) * HG;
+  static constexpr uint32_t kColOnes = kColL + HG;
+  static_assert(HG > 64 || kColOnes + 8 <= kTmemCols, "TMEM columns");
   static constexpr int kSmem = 1024 + kNumChunks * kChunkBytes + kQBytes + (int)sizeof(Ctrl);
   static constexpr uint32_t kPRowBytes = 2 * HG;  // P^T tile row (one token, HG fp16)
 };
@@ -789,27 +793,6 @@ struct Cols {
 };
 
 
-// Sum over the warp's 32 lanes of each of W values; lane l returns the total
-// of element l >> 1 (W = 16) or l >> 2 (W = 8), by recursive halving.
-template <int W>
-__device__ __forceinline__ float warp_colsum(float (&v)[W], int lane) {
-#pragma unroll
-  for (int s = 16, n = W / 2; n >= 1; s >>= 1, n >>= 1) {
-    const bool hi = (lane & s) != 0;
-#pragma unroll
-    for (int i = 0; i < n; ++i) {
-      const float send = hi ? v[i] : v[i + n];
-      const float keep = hi ? v[i + n] : v[i];
-      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, s);
-    }
-  }
-  float t = v[0];
-  constexpr int kRest = W == 16 ? 1 : 2;  // lanes still holding partial sums of one element
-#pragma unroll
-  for (int s = kRest; s >= 1; s >>= 1) t += __shfl_xor_sync(0xffffffffu, t, s);
-  return t;
-}
-
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -920,25 +903,36 @@ struct SegEnd {
   size_t pidx;  // partial slot (CTA index + unit)
 };
 
-// Segment end: l[h] = sum of the four row quarters' sums, then out = O / l
-// (or the partial o, m, l) for this warp's heads, then release O^T to the next
-// segment. lsum[c] holds, in the lanes that warp_colsum leaves it in, this
-// warp's sum over its 32 rows and the segment's tiles of head column group c.
+// Segment end: l[h] from the row-sum accumulator (every TMEM lane holds the
+// same sums; the warps of lane quarter 0 read theirs once the segment's last
+// row-sum MMAs, phase rs_parity of rs_done, have completed), then out = O / l
+// (or the partial o, m, l) for this warp's heads, then release O^T and the
+// row sums to the next segment.
 template <int CB, int HG>
 __device__ bool epilogue(const Params& p, const SegEnd& e, Ctrl& ctl, uint32_t tmem, uint32_t& gph,
-                         const float (&lsum)[Cols<HG>::kN], int warp, int lane) {
+                         uint32_t rs_parity, int warp, int lane) {
   using C = Cols<HG>;
   const int q4 = warp & 3, half = warp >> 2, row = q4 * 32 + lane, cb0 = half * C::kPerWarp;
   const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
   const uint32_t t_o = tmem + cb0 + lane_off;
-  constexpr int kSh = C::kW == 16 ? 1 : 2;
+  if (q4 == 0) {
+    if (!wwait(&ctl.rs_done, rs_parity, ctl, kSitePvEpi, p.dev_err)) return false;
+    tc_fence_after();
 #pragma unroll
-  for (int c = 0; c < C::kN; ++c)
-    if ((lane & ((1 << kSh) - 1)) == 0) ctl.red[q4][cb0 + c * C::kW + (lane >> kSh)] = lsum[c];
+    for (int c = 0; c < C::kN; ++c) {
+      uint32_t r[C::kW];
+      tmem_ld(tmem + Cfg<HG>::kColL + cb0 + c * C::kW, r);
+      tmem_ld_wait();
+      if (lane == 0) {
+#pragma unroll
+        for (int jj = 0; jj < C::kW; ++jj) ctl.red[0][cb0 + c * C::kW + jj] = __uint_as_float(r[jj]);
+      }
+    }
+  }
   if (!group_sync(ctl, gph, p.dev_err)) return false;
   const int tid = threadIdx.x;  // 0 .. 255 over the worker warps
   if (tid < HG) {
-    const float l = (ctl.red[0][tid] + ctl.red[1][tid]) + (ctl.red[2][tid] + ctl.red[3][tid]);
+    const float l = ctl.red[0][tid];
     ctl.alpha[tid] = l;
     ctl.inv[tid] = l > 0.0f ? 1.0f / l : 0.0f;  // one division per head; 0 for a head that saw no key
   }
@@ -1039,11 +1033,6 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
   bool ok = true;
   bool pending = false;  // the previous tile ended a segment whose epilogue is still due
   SegEnd pend{};
-  // Row sums of P for the current segment: per head column group, the warp's
-  // column sum over its 32 rows (warp_colsum layout), accumulated over tiles.
-  float lsum[C::kN], lsum_done[C::kN];  // lsum_done: the pending segment's sums
-#pragma unroll
-  for (int c = 0; c < C::kN; ++c) lsum[c] = lsum_done[c] = 0.0f;
 
   // Packed rows of the tile about to be dequantised (INT4/INT2), fetched a tile ahead.
   Fetch f[kMyChunks];
@@ -1144,6 +1133,9 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       // (this library's block: content chunks 2 kc + par, then half par of the RoPE chunk)
       const int k = kEarly && kc == 4 ? 8 : 2 * kc + par;
       if (k >= kNumChunks) break;
+      // The RoPE chunk's slot held the previous tile's P, which its row-sum
+      // MMAs (committed apart from the PV) may still be reading.
+      if (k == 8 && !(ok = wwait(&ctl.rs_done, (it & 1u) ^ 1u, ctl, kSiteDqSlot, p.dev_err))) break;
       if constexpr (CB == 16) {
         // (a wait per chunk, as a scheduling barrier: without it the compiler
         // hoists the loads of later chunks and spills)
@@ -1199,7 +1191,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     // ---- the previous segment's results (its last PV completed: pv_done was waited for above)
     if (pending) {
       tc_fence_after();
-      if (!(ok = epilogue<CB, HG>(p, pend, ctl, tmem, gph, lsum_done, warp, lane))) break;
+      if (!(ok = epilogue<CB, HG>(p, pend, ctl, tmem, gph, (it - 1) & 1u, warp, lane))) break;
       pending = false;
       if (lane == 0 && warp == 0) QMLA_TRACE(20, it);
     }
@@ -1249,12 +1241,12 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       }
       if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
       if (!ti.first) {
-        constexpr int kSh = C::kW == 16 ? 1 : 2;
+        // (the previous tile's row-sum MMAs must have landed before L is rescaled)
+        if (!(ok = wwait(&ctl.rs_done, (it - 1) & 1u, ctl, kSitePvEpi, p.dev_err))) break;
+        tc_fence_after();
 #pragma unroll
-        for (int c = 0; c < C::kN; ++c) lsum[c] *= ctl.alpha[cb0 + c * C::kW + (lane >> kSh)];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {  // O^T blocks 0..3
-          const uint32_t col = i * HG;
+        for (int i = 0; i < 5; ++i) {  // O^T blocks 0..3 and the row sums
+          const uint32_t col = i < 4 ? i * HG : Cfg<HG>::kColL;
 #pragma unroll
           for (int c = 0; c < C::kN; ++c) {
             uint32_t r[C::kW];
@@ -1275,24 +1267,9 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
       mbar_arrive_if(lane == 0 ? 1u : 0u, &ctl.p_fixed);
       ++nresc;
     }
-    // Row sums of the fp16 weights the PV MMA multiplies with: this warp's column
-    // sums over its 32 rows, added to the segment's running sums in registers.
-#pragma unroll
-    for (int c = 0; c < C::kN; ++c) {
-      float v[C::kW];
-#pragma unroll
-      for (int jj = 0; jj < C::kW; jj += 2) {
-        const float2 pf = __half22float2(*reinterpret_cast<const __half2*>(&pk[c * (C::kW / 2) + (jj >> 1)]));
-        v[jj] = pf.x;
-        v[jj + 1] = pf.y;
-      }
-      const float t = warp_colsum<C::kW>(v, lane);
-      lsum[c] = ti.first ? t : lsum[c] + t;
-    }
+    // (the row sums of the fp16 weights are summed by the tensor core, see mma_issuer)
     if (lane == 0 && warp == 0) QMLA_TRACE(18, it);
     if (ti.last) {
-#pragma unroll
-      for (int c = 0; c < C::kN; ++c) lsum_done[c] = lsum[c];
       pending = true;
       pend.b = ti.b;
       pend.hg = ti.hg;
@@ -1305,7 +1282,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
   if (ok && pending) {
     if ((ok = wwait(&ctl.pv_done, (it - 1) & 1u, ctl, kSitePvEpi, p.dev_err))) {
       tc_fence_after();
-      ok = epilogue<CB, HG>(p, pend, ctl, tmem, gph, lsum_done, warp, lane);
+      ok = epilogue<CB, HG>(p, pend, ctl, tmem, gph, (it - 1) & 1u, warp, lane);
     }
   }
   if (!ok && lane == 0) set_abort(ctl, p.dev_err);
@@ -1343,6 +1320,7 @@ __device__ void mma_issuer(const Params& p, Sched sc, uint32_t chunks, uint8_t* 
                            int j) {
   constexpr uint32_t kIdQK = idesc_f16_f32(128, HG, false, false);
   constexpr uint32_t kIdPV = idesc_f16_f32(128, HG, true, true);
+  constexpr uint32_t kIdL = idesc_f16_f32(128, HG, false, true);  // A (ones) from TMEM, B = P^T
   constexpr uint32_t kRB = Cfg<HG>::kPRowBytes;
   constexpr uint32_t kSboP = 8 * kRB;
   constexpr int kSteps = 4 / kQkParts;  // QK K-steps per chunk and issuer
@@ -1410,6 +1388,17 @@ __device__ void mma_issuer(const Params& p, Sched sc, uint32_t chunks, uint8_t* 
       umma_f16_ss(t_o, pv_a0 + static_cast<uint64_t>((kk * 2048) >> 4),
                   pv_b0 + static_cast<uint64_t>((kk * 2 * kSboP) >> 4), kIdPV, kk == 0 ? acc0 : 1u);
     umma_commit(&ctl.pv_done);
+    if (j == kIssuers - 1) {
+      // Row sums of P: L[m, h] += sum_t 1 * P^T[t, h] for every row m, with an
+      // all-ones A operand in TMEM. Committed on their own barrier so that the
+      // PV completion the dequantisation waits for does not wait for them; they
+      // run while the next tile's first chunks are written.
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk)
+        umma_f16_ts(tmem + Cfg<HG>::kColL, tmem + Cfg<HG>::kColOnes,
+                    pv_b0 + static_cast<uint64_t>((kk * 2 * kSboP) >> 4), kIdL, kk == 0 ? acc0 : 1u);
+      umma_commit(&ctl.rs_done);
+    }
     QMLA_TRACE(24 + j, it);
     if (j == 0) QMLA_TRACE(15, it);
     ++it;
@@ -1445,6 +1434,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
     for (int k = 0; k < kNumChunks; ++k) mbar_init(&ctl.chunk_full[k], k == 8 && (CB == 4 || CB == 2) ? 8 : 4);
     mbar_init(&ctl.pv_done, kIssuers);
     mbar_init(&ctl.s_full, kQkParts);
+    mbar_init(&ctl.rs_done, 1);
     mbar_init(&ctl.p_full, kWorkers);
     mbar_init(&ctl.p_fixed, kWorkers);
     ctl.resc_tile = 0u;
@@ -1463,6 +1453,16 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = ctl.tmem_base;
+  if (warp < 4) {  // the all-ones A operand of the row-sum MMAs, each warp its lane quarter
+    uint32_t r[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) r[i] = 0x3c003c00u;  // fp16 pair (1, 1)
+    tmem_st(tmem + (static_cast<uint32_t>(warp * 32) << 16) + Cfg<HG>::kColOnes, r);
+    tmem_st_wait();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
   if (warp >= kWorkers && lane != 0) return;  // each MMA role is a single thread
   // The set-up above may overlap the prep kernel; everything below reads what
   // prep and the cache writer before it produced.
