@@ -1119,11 +1119,16 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
 
     // ---- dequantise this tile. The previous tile's four PV blocks (one issuer
     // each) complete together, so one wait frees every slot. For this
-    // library's INT4 / INT2 block (protected rows included) the first chunk's
-    // arithmetic runs before that wait and each further chunk's while the
-    // stores of the one before drain, ahead of its proxy fence.
+    // library's INT4 / INT2 block (protected rows included) the arithmetic of
+    // the first chunk and of the RoPE half runs before that wait and each
+    // further chunk's while the stores of the one before drain, ahead of its
+    // proxy fence.
     uint32_t dq[kEarly ? 32 : 1];
-    if constexpr (kEarly) row_regs<CB, PROT>(dq, f[0], par, psrc_cur);
+    uint32_t dqh[kEarly ? 32 : 1];  // the RoPE half (16 words), also computed before the wait
+    if constexpr (kEarly) {
+      row_regs<CB, PROT>(dq, f[0], par, psrc_cur);
+      row_regs_half<PROT>(dqh, f[4], psrc_cur, par);
+    }
     if (lane == 0 && warp == 0) QMLA_TRACE(105, it);
     if (!(ok = wwait(&ctl.pv_done, (it & 1u) ^ 1u, ctl, kSiteDqSlot, p.dev_err))) break;
     if (lane == 0) QMLA_TRACE(88 + warp, it);
@@ -1154,14 +1159,10 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
         if (kc < 4) {
           store_regs(chunks + k * kChunkBytes, row, dq);
         } else {
-          store_half(chunks + 8 * kChunkBytes, row, dq, par);
+          store_half(chunks + 8 * kChunkBytes, row, dqh, par);
         }
         // the next chunk's arithmetic while these stores drain
-        if (kc + 1 < 4) {
-          row_regs<CB, PROT>(dq, f[kc + 1], k + 2, psrc_cur);
-        } else if (kc + 1 == 4) {
-          row_regs_half<PROT>(dq, f[4], psrc_cur, par);
-        }
+        if (kc + 1 < 4) row_regs<CB, PROT>(dq, f[kc + 1], k + 2, psrc_cur);
       } else {
         dq_row<CB, PROT>(chunks + k * kChunkBytes, row, k, psrc_cur, f[kc]);
         f[kc] = fetch_chunk<CB>(blk_nx, valid_nx, k, slot);  // the next tile's rows of this chunk
