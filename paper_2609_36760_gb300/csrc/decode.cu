@@ -440,7 +440,12 @@ __device__ __forceinline__ Fetch fetch_rope_half(const uint8_t* blk, bool valid,
   if (!valid) return f;
   using L = BlockLayout<CB>;
   f.a = ldg_nc_v4(blk + L::code_off(8, slot) + 16 * h);
-  f.sz = ldg_nc_u32(blk + L::sz_off(8, slot));
+  if constexpr (CB == kC4R4) {
+    f.sz = ldg_nc_u32(blk + L::pe_scale_off(slot));  // the fp32 RoPE scale
+    f.z = ldg_nc_u8(blk + L::zero_off(8, slot));
+  } else {
+    f.sz = ldg_nc_u32(blk + L::sz_off(8, slot));
+  }
   return f;
 }
 
@@ -612,6 +617,51 @@ __device__ __forceinline__ void store_row_c4r4(uint32_t chunk_base, int row, con
   }
 }
 
+// The paper's page into registers (the decode workers compute a chunk row
+// before its stores, as dq_regs does for this library's block): NW code words
+// of f (8 for a row, 4 for half a RoPE row) into o[0 .. 4 NW). Same arithmetic
+// as store_row_c4r4: fp16 subtract-and-multiply for a content row whose bf16
+// scale is an fp16 value, else (the RoPE key, or a content scale outside
+// fp16's normal range) the fp32 product rounded once to fp16.
+template <int NW>
+__device__ __forceinline__ void dq_regs_c4r4(uint32_t (&o)[32], const Fetch& f, bool content) {
+  const float s = __uint_as_float(f.sz);
+  const __half2 zz2 = __half2half2(__float2half_rn(1024.0f + static_cast<float>(f.z)));
+  const uint32_t zz = *reinterpret_cast<const uint32_t*>(&zz2);
+  constexpr uint32_t K = 0x64646464u;
+  const uint32_t w[8] = {f.a.x, f.a.y, f.a.z, f.a.w, f.b.x, f.b.y, f.b.z, f.b.w};
+  const __half sh = __float2half_rn(s);
+  if (content && __half2float(sh) == s) {
+    const __half2 s2 = __half2half2(sh);
+    const uint32_t ss = *reinterpret_cast<const uint32_t*>(&s2);
+#pragma unroll
+    for (int i = 0; i < NW; ++i) {
+      const uint32_t lo = w[i] & 0x0F0F0F0Fu;
+      const uint32_t hi = (w[i] >> 4) & 0x0F0F0F0Fu;
+      o[4 * i + 0] = dq2(__byte_perm(lo, K, 0x4140), zz, ss);
+      o[4 * i + 1] = dq2(__byte_perm(hi, K, 0x4140), zz, ss);
+      o[4 * i + 2] = dq2(__byte_perm(lo, K, 0x4342), zz, ss);
+      o[4 * i + 3] = dq2(__byte_perm(hi, K, 0x4342), zz, ss);
+    }
+  } else {
+    auto dqf = [&](uint32_t x) {
+      uint32_t t;
+      asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(t) : "r"(x), "r"(zz));
+      const float2 d = __half22float2(*reinterpret_cast<const __half2*>(&t));
+      return pack_h2(d.x * s, d.y * s);
+    };
+#pragma unroll
+    for (int i = 0; i < NW; ++i) {
+      const uint32_t lo = w[i] & 0x0F0F0F0Fu;
+      const uint32_t hi = (w[i] >> 4) & 0x0F0F0F0Fu;
+      o[4 * i + 0] = dqf(__byte_perm(lo, K, 0x4140));
+      o[4 * i + 1] = dqf(__byte_perm(hi, K, 0x4140));
+      o[4 * i + 2] = dqf(__byte_perm(lo, K, 0x4342));
+      o[4 * i + 3] = dqf(__byte_perm(hi, K, 0x4342));
+    }
+  }
+}
+
 // A protected row's chunk k: 64 bf16 values (8 x 16 bytes) rounded to fp16 and
 // placed in the same within-piece channel order as the packed rows
 // (bf16 -> fp16 is exact for magnitudes in [2^-14, 65504]).
@@ -652,11 +702,10 @@ __device__ __forceinline__ void store_row_bf16(uint32_t chunk_base, int row, con
   }
 }
 
-// One row's chunk k of this library's block as dq_row would store it (the
-// eight 16-byte pieces in order), computed into registers: the protected bf16
-// row when ps is set, else the packed row f. The decode workers compute it
-// before waiting for the chunk's slot, so only the stores follow the slot's
-// release.
+// One row's chunk k of a packed cache (this library's block or the paper's
+// page) as dq_row would store it (the eight 16-byte pieces in order),
+// computed into registers: the protected bf16 row when ps is set, else the
+// packed row f. The decode workers compute it ahead of its stores.
 template <int CB, bool PROT>
 __device__ __forceinline__ void row_regs(uint32_t (&o)[32], const Fetch& f, int k, const uint8_t* ps) {
   if (PROT && ps != nullptr) {
@@ -680,6 +729,8 @@ __device__ __forceinline__ void row_regs(uint32_t (&o)[32], const Fetch& f, int 
         for (int e = 0; e < 4; ++e) o[4 * i + e] = pack_h2(v[Perm<4>::at(2 * e)], v[Perm<4>::at(2 * e + 1)]);
       }
     }
+  } else if constexpr (CB == kC4R4) {
+    dq_regs_c4r4<8>(o, f, k < 8);
   } else {
     dq_regs(o, f, CB == 4 || k == 8);
   }
@@ -691,7 +742,7 @@ __device__ __forceinline__ void row_regs(uint32_t (&o)[32], const Fetch& f, int 
 // Half h of a RoPE-key row into o[0..15] (pieces 4 h .. 4 h + 3): the
 // protection row's bf16 channels 32 h .. 32 h + 31 rounded to fp16 when the
 // row is protected, else dq_half of the packed codes.
-template <bool PROT>
+template <int CB, bool PROT>
 __device__ __forceinline__ void row_regs_half(uint32_t (&o)[32], const Fetch& f, const uint8_t* ps, int h) {
   if (PROT && ps != nullptr) {
     uint4 pv[4];
@@ -709,6 +760,8 @@ __device__ __forceinline__ void row_regs_half(uint32_t (&o)[32], const Fetch& f,
 #pragma unroll
       for (int e = 0; e < 4; ++e) o[4 * i + e] = pack_h2(v[Perm<4>::at(2 * e)], v[Perm<4>::at(2 * e + 1)]);
     }
+  } else if constexpr (CB == kC4R4) {
+    dq_regs_c4r4<4>(o, f, false);
   } else {
     dq_half(o, f);
   }
@@ -1025,9 +1078,10 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
   const uint32_t ptile = chunks + 8 * kChunkBytes;
   const float sl2 = p.scale_log2;
   constexpr int kMyChunks = 5;  // chunk steps per warp (the paper's page and BF16: parity 1 has 4)
-  // This library's INT4 / INT2 block: each warp dequantises 4 content chunks
-  // and half of the RoPE-key chunk (channels 32 par .. 32 par + 31).
-  constexpr bool kEarly = CB == 4 || CB == 2;
+  // The packed caches (this library's INT4 / INT2 block and the paper's page):
+  // each warp dequantises 4 content chunks and half of the RoPE-key chunk
+  // (channels 32 par .. 32 par + 31), each row's arithmetic ahead of its stores.
+  constexpr bool kEarly = CB == 4 || CB == 2 || CB == kC4R4;
   uint32_t it = 0, gph = 0, nresc = 0;
   int seg_j0 = 0;
   bool ok = true;
@@ -1118,16 +1172,15 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     if (lane == 0 && warp == 0) QMLA_TRACE(0, it);
 
     // ---- dequantise this tile. The previous tile's four PV blocks (one issuer
-    // each) complete together, so one wait frees every slot. For this
-    // library's INT4 / INT2 block (protected rows included) the arithmetic of
-    // the first chunk and of the RoPE half runs before that wait and each
-    // further chunk's while the stores of the one before drain, ahead of its
-    // proxy fence.
+    // each) complete together, so one wait frees every slot. For the packed
+    // caches (protected rows included) the arithmetic of the first chunk and
+    // of the RoPE half runs before that wait and each further chunk's while
+    // the stores of the one before drain, ahead of its proxy fence.
     uint32_t dq[kEarly ? 32 : 1];
     uint32_t dqh[kEarly ? 32 : 1];  // the RoPE half (16 words), also computed before the wait
     if constexpr (kEarly) {
       row_regs<CB, PROT>(dq, f[0], par, psrc_cur);
-      row_regs_half<PROT>(dqh, f[4], psrc_cur, par);
+      row_regs_half<CB, PROT>(dqh, f[4], psrc_cur, par);
     }
     if (lane == 0 && warp == 0) QMLA_TRACE(105, it);
     if (!(ok = wwait(&ctl.pv_done, (it & 1u) ^ 1u, ctl, kSiteDqSlot, p.dev_err))) break;
@@ -1135,7 +1188,7 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     if (lane == 0 && (warp & 3) == 0) QMLA_TRACE(warp == 0 ? 96 : 101, it);
 #pragma unroll
     for (int kc = 0; kc < kMyChunks; ++kc) {
-      // (this library's block: content chunks 2 kc + par, then half par of the RoPE chunk)
+      // (packed caches: content chunks 2 kc + par, then half par of the RoPE chunk)
       const int k = kEarly && kc == 4 ? 8 : 2 * kc + par;
       if (k >= kNumChunks) break;
       // The RoPE chunk's slot held the previous tile's P, which its row-sum
@@ -1430,9 +1483,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_main(const Params p) {
   }
 
   if (threadIdx.x == 0) {
-    // chunk k is written by the 4 warps of its parity; this library's INT4 /
-    // INT2 block splits the RoPE chunk (k = 8) over all 8 workers
-    for (int k = 0; k < kNumChunks; ++k) mbar_init(&ctl.chunk_full[k], k == 8 && (CB == 4 || CB == 2) ? 8 : 4);
+    // chunk k is written by the 4 warps of its parity; the packed caches split
+    // the RoPE chunk (k = 8) over all 8 workers
+    for (int k = 0; k < kNumChunks; ++k) mbar_init(&ctl.chunk_full[k], k == 8 && CB != 16 ? 8 : 4);
     mbar_init(&ctl.pv_done, kIssuers);
     mbar_init(&ctl.s_full, kQkParts);
     mbar_init(&ctl.rs_done, 1);
