@@ -16,14 +16,14 @@
 //                                   dequantise RN_f16(s (q - z)) into nine
 //                                   swizzled fp16 chunks of 128 tokens x 64
 //                                   channels in shared memory;
-//                    MMA thread     S^T[t,h] = C_hat[t,:] . q[h,:] over 576
+//                    MMA issuers    S^T[t,h] = C_hat[t,:] . q[h,:] over 576
 //                                   channels (tcgen05, M=128 tokens, N=HG,
 //                                   K-major A and B) into TMEM;
 //                    softmax warps  read S^T from TMEM (one token per thread),
 //                                   keep a per-head reference max (rescaling O
 //                                   only when a score exceeds it by 2^8), write
 //                                   P^T = 2^(S*scale*log2e - m) as fp16;
-//                    MMA thread     O^T[c,h] += C_hat[:,c]^T P^T (M = 128
+//                    MMA issuers    O^T[c,h] += C_hat[:,c]^T P^T (M = 128
 //                                   channels x 4, N=HG, K = 128 tokens; the same
 //                                   shared-memory chunks read MN-major).
 //                  The reconstructed content tile serves both QK and PV and a
@@ -1274,14 +1274,14 @@ __device__ void worker_role(const Params& p, Sched sc, uint32_t chunks, Ctrl& ct
     __syncwarp();
     mbar_arrive_if(lane == 0 ? 1u : 0u, &ctl.p_full);
     if (lane == 0 && warp == 0) QMLA_TRACE(19, it);
-    // Off the MMA thread's path from here: learn whether any warp asked for a rescale.
+    // Off the MMA issuers' path from here: learn whether any warp asked for a rescale.
     if (!(ok = wwait(&ctl.p_full, it & 1u, ctl, kSiteGrp, p.dev_err))) break;
     if (lane == 0 && warp == 0) QMLA_TRACE(17, it);
     if (*reinterpret_cast<volatile uint32_t*>(&ctl.resc_tile) == it + 1) {
       // Raise the reference to the running max; O and the row sums were
       // accumulated against the old one and are scaled by alpha = 2^(m_old - m_new).
       // The previous PV has completed (its slots were waited for above); the
-      // MMA thread waits on p_fixed before this tile's PV.
+      // MMA issuers wait on p_fixed before this tile's PV.
       tc_fence_after();
       warp_tile_max<HG>(t_s, sl2, lim, &ctl.red[q4][cb0], lane);
       if (!(ok = group_sync(ctl, gph, p.dev_err))) break;
