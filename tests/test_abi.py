@@ -142,7 +142,7 @@ def test_static_decode_host_checks(libqmla):
     fake = ctypes.c_void_p(0x10000)
     base = [fake, 4, 4, fake, fake, 1, 16, fake, 1, fake, 0.1, fake, None, None, None]
     for i, bad in ((1, 3), (1, 8), (6, 0), (6, 129), (5, 0), (0, None), (3, None), (7, None), (9, None),
-                   (11, None), (10, -1.0), (10, 0.0), (0, ctypes.c_void_p(0x10008)),
+                   (11, None), (10, -1.0), (10, 0.0), (0, ctypes.c_void_p(0x10008)), (0, ctypes.c_void_p(0x10010)),
                    (3, ctypes.c_void_p(0x10004)), (11, ctypes.c_void_p(0x10004)), (8, 1 << 26)):
         args = list(base)
         args[i] = bad

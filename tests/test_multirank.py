@@ -64,3 +64,4 @@ def test_two_ranks_gloo():
 def test_single_process_helpers():
     assert bench.max_over_ranks(0.25, None, "cpu") == 0.25
     assert bench.whole_job_value(1, 500.0, 0.5) == pytest.approx(1e6)
+
