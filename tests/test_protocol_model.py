@@ -18,9 +18,12 @@ Checked at every step:
 Mutations (each wait taken out in turn, among them the P slot reused without
 waiting for the row-sum MMAs, the race a full-size two-token GPU test
 exposed) must be caught, except two that the model shows implied by other
-waits on this path: the rescale's row-sum wait (needed on the BF16 cache,
-whose RoPE chunk only one parity stores, so the other parity has not waited)
-and the issuers' o_free wait (kept as an explicit guard)."""
+waits, kept as explicit guards: the rescale's row-sum wait (the P hand-off
+comes after every worker's, or on the BF16 cache every parity-0 worker's,
+row-sum wait before the RoPE chunk's store) and the issuers' o_free wait (the
+issuers wait for every worker's P, written after its epilogue). On the BF16
+cache, where one parity stores the RoPE chunk, the epilogue's row-sum wait is
+needed."""
 import random
 
 import pytest
@@ -37,8 +40,11 @@ class Hazard(AssertionError):
 
 
 class Sim:
-    def __init__(self, n_tiles, last, resc, seed, drop=None):
+    def __init__(self, n_tiles, last, resc, seed, drop=None, bf16=False):
         self.rng = random.Random(seed)
+        # how often the tensor core and the copy engine get to finish work,
+        # against the threads' steps: some runs have a very slow tensor core
+        self.async_weight = self.rng.choice([1.0, 0.3, 0.05])
         self.n = n_tiles
         self.last = last  # last[t]: tile t ends a segment
         self.first = [t == 0 or last[t - 1] for t in range(n_tiles)]
@@ -50,10 +56,13 @@ class Sim:
                 u += 1
         self.resc = resc  # resc[t]: the softmax of tile t raises the reference
         self.drop = drop  # the name of one wait to leave out (a mutation), or None
+        # bf16: the BF16-cache path, whose workers store chunks 2 kc + parity for
+        # kc = 0..4 (the RoPE chunk 8 by parity 0 only), each after a PV wait
+        self.bf16 = bf16
         self.bars = {"pv_done": Bar(4), "rs_done": Bar(1), "s_full": Bar(2), "p_full": Bar(8),
                      "p_fixed": Bar(8), "o_free": Bar(8), "q_full": Bar(1), "grp": Bar(8)}
         for k in range(9):
-            self.bars["chunk%d" % k] = Bar(8 if k == 8 else 4)
+            self.bars["chunk%d" % k] = Bar(8 if k == 8 and not bf16 else 4)
         self.parts = {}  # (buffer, version) -> set of writer parts
         self.state = {}  # accumulator / copied buffer -> completed version
         self.fifo = {j: [] for j in range(4)}  # per issuer: in-order async ops
@@ -77,14 +86,29 @@ class Sim:
         for t in range(self.n):
             if self.drop != "worker_pv":
                 yield ("wait", "pv_done", t - 1)  # the previous tile's PV has released every slot
-            for kc in range(4):
-                k = 2 * kc + par
-                yield ("write", "slot%d" % k, t, q4)
-                yield ("arrive", "chunk%d" % k)
-            if self.drop != "rope_rs":
-                yield ("wait", "rs_done", t - 1)  # the slot held P, read by the row-sum MMAs
-            yield ("write", "slot8", ("rope", t), w)
-            yield ("arrive", "chunk8")
+            if self.bf16:
+                for kc in range(5):
+                    k = 2 * kc + par
+                    if k > 8:
+                        break
+                    if k == 8 and self.drop != "rope_rs":
+                        yield ("wait", "rs_done", t - 1)
+                    if kc > 0 and self.drop != "worker_pv":
+                        yield ("wait", "pv_done", t - 1)
+                    if k == 8:
+                        yield ("write", "slot8", ("rope", t), q4)
+                    else:
+                        yield ("write", "slot%d" % k, t, q4)
+                    yield ("arrive", "chunk%d" % k)
+            else:
+                for kc in range(4):
+                    k = 2 * kc + par
+                    yield ("write", "slot%d" % k, t, q4)
+                    yield ("arrive", "chunk%d" % k)
+                if self.drop != "rope_rs":
+                    yield ("wait", "rs_done", t - 1)  # the slot held P, read by the row-sum MMAs
+                yield ("write", "slot8", ("rope", t), w)
+                yield ("arrive", "chunk8")
             if pending is not None:  # the previous segment's results
                 e = pending
                 if q4 == 0:
@@ -143,7 +167,7 @@ class Sim:
                 for k in range(9):
                     if self.drop != "chunk":
                         yield ("wait", "chunk%d" % k, t)
-                    src = ("slot8", ("rope", t), 8) if k == 8 else ("slot%d" % k, t, 4)
+                    src = ("slot8", ("rope", t), 4 if self.bf16 else 8) if k == 8 else ("slot%d" % k, t, 4)
                     yield ("mma", j, [src, ("Q", self.unit[t], None)], ["S%d" % j], t)
                 yield ("commit", j, "s_full")
             if self.drop != "issuer_p_full":
@@ -265,15 +289,19 @@ class Sim:
                         self.start(a, self.cur[a])
                     except StopIteration:
                         self.actors[a] = None
-            choices = [("a", a) for a, op in self.cur.items() if op is not None and self.enabled(op)]
-            choices += [("q", j) for j in range(4) if self.fifo[j]]
+            threads = [("a", a) for a, op in self.cur.items() if op is not None and self.enabled(op)]
+            engines = [("q", j) for j in range(4) if self.fifo[j]]
             if self.copies:
-                choices.append(("q", "copy"))
-            if not choices:
+                engines.append(("q", "copy"))
+            if not threads and not engines:
                 if any(op is not None for op in self.cur.values()):
                     raise Hazard(f"deadlock: {[(a, op) for a, op in self.cur.items() if op is not None]}")
                 return
-            kind, who = self.rng.choice(choices)
+            if engines and (not threads or self.rng.random() < self.async_weight * len(engines) /
+                            (len(engines) + len(threads))):
+                kind, who = self.rng.choice(engines)
+            else:
+                kind, who = self.rng.choice(threads)
             if kind == "a":
                 op, self.cur[who] = self.cur[who], None
                 self.execute(who, op)
@@ -324,3 +352,33 @@ def test_waits_implied_on_the_packed_path(drop):
         n, last, resc = list(_patterns())[pattern]
         for seed in range(60):
             Sim(n, last, resc, seed, drop=drop).run()
+
+
+@pytest.mark.parametrize("pattern", list(range(4)))
+def test_bf16_path_has_no_hazard(pattern):
+    n, last, resc = list(_patterns())[pattern]
+    for seed in range(100):
+        Sim(n, last, resc, seed, bf16=True).run()
+
+
+@pytest.mark.parametrize("drop", ["rope_rs", "epi_rs", "worker_pv", "s_full", "chunk"])
+def test_bf16_path_needs_its_waits(drop):
+    # On the BF16 cache the RoPE chunk is stored by parity 0 only, so the
+    # parity-1 warps reach the epilogue without having waited for the row-sum
+    # MMAs: the epilogue's wait is needed there.
+    caught = 0
+    for pattern in range(4):
+        n, last, resc = list(_patterns())[pattern]
+        for seed in range(60):
+            try:
+                Sim(n, last, resc, seed, drop=drop, bf16=True).run()
+            except Hazard:
+                caught += 1
+    assert caught > 0, drop
+
+
+def test_rescale_wait_implied_on_the_bf16_path():
+    for pattern in range(4):
+        n, last, resc = list(_patterns())[pattern]
+        for seed in range(60):
+            Sim(n, last, resc, seed, drop="resc_rs", bf16=True).run()
